@@ -1,0 +1,412 @@
+"""Benchmark of the GB300 dense GEMM library (C = A.B, int8->int32 exact and
+bf16->fp32->bf16 RNE).
+
+One step = every GEMM of the chosen workload once (default: the square sweep
+M=N=K in {512,1024,2048,4096}, int8 and bf16, B column-major).  Inputs are
+seeded synthetic matrices (workloads.py) resident in HBM before timing.  L2
+(129 MB) is flushed by writing a 512 MiB buffer before every timed GEMM; each
+GEMM is bracketed by CUDA events on its stream, so flushes are not timed.
+
+  value       whole-job throughput, sum(2*M*N*K) / sum(event time), in TOPS
+              (tera-ops/s; int8 MACs and bf16 FMAs both count 2 ops)
+  e2e         the same through the C ABI from pinned HOST buffers: H2D copies
+              of A and B, the GEMM, D2H of C, all inside the timed events
+  roofline    the dominant kernel (largest share of step time): the
+              tensor-core kernel of one GEMM, timed alone through the
+              library's profiling events, against the measured bf16 peak
+  cpu_baseline  the CPU oracle on a bounded sample (whole rows of C) of the
+              same GEMMs, on this host's cores
+
+``--impl reference`` times the CPU oracle itself (the only reference this
+path has) on bounded samples of the same workload.
+
+Multi-GPU (torchrun): every rank runs the same workload on its own GPU
+(replicas; the GEMM has no exchange step), value = all ranks' ops / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2512_13282_gb300 import workloads as W  # noqa: E402
+
+METRIC = "int8 TOPS & bf16 TFLOPS per GEMM shape, 1 GB300; % of dense tensor-core peak"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FLUSH_BYTES = 512 << 20
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK), "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons in the background."""
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        self.lines += [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        rows = []
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 8:
+                continue
+            if self.uuid and f[0] != self.uuid and not self.uuid.endswith(f[0]) and not f[0].endswith(self.uuid):
+                continue
+            try:
+                rows.append((float(f[1]), float(f[2]), f[4:8]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i in range(4) if r[i].lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# -------------------------------------------------------------- our path
+
+class GemmCase:
+    def __init__(self, g: W.Gemm, dev):
+        from paper_2512_13282_gb300 import gemm as G
+        self.g, self.G = g, G
+        A, B = W.make_inputs(g)
+        if g.dtype == "int8":
+            ha, hb = torch.from_numpy(A), torch.from_numpy(B)
+            self.C = torch.empty((g.M, g.N), dtype=torch.int32, device=dev)
+            self.fn = G.gemm_s8s8_s32
+        else:
+            ha, hb = torch.from_numpy(A.view(np.int16)), torch.from_numpy(B.view(np.int16))
+            self.C = torch.empty((g.M, g.N), dtype=torch.int16, device=dev)
+            self.fn = G.gemm_bf16_f32acc_bf16
+        self.A, self.B = ha.to(dev), hb.to(dev)
+        self.hA, self.hB = ha.pin_memory(), hb.pin_memory()
+        self.hC = torch.empty(self.C.shape, dtype=self.C.dtype).pin_memory()
+        self.ldb = g.N if g.layout == W.B_ROW_MAJOR else g.K
+        self.h2d = self.hA.numel() * self.hA.element_size() + self.hB.numel() * self.hB.element_size()
+        self.d2h = self.hC.numel() * self.hC.element_size()
+
+    def launch(self, A=None, B=None, C=None):
+        g = self.g
+        st = self.fn(g.M, g.N, g.K, self.A if A is None else A, g.K, self.B if B is None else B, self.ldb,
+                     g.layout, self.C if C is None else C, g.N, None)
+        if st != 0:
+            raise RuntimeError(f"{g.name}: {self.G.gemm_status_string(st)}")
+
+    def launch_e2e(self):
+        self.A.copy_(self.hA, non_blocking=True)
+        self.B.copy_(self.hB, non_blocking=True)
+        self.launch()
+        self.hC.copy_(self.C, non_blocking=True)
+
+
+def run_ours(args, rank, world, dev):
+    from paper_2512_13282_gb300 import build as Bld
+    from paper_2512_13282_gb300 import gemm as G
+    Bld.build()
+    G.library()
+    wl = W.WORKLOADS[args.workload]
+    cases = [GemmCase(g, dev) for g in wl.gemms]
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(times=None, kern=None):
+        for i, c in enumerate(cases):
+            flush.fill_(float(i))
+            if times is not None:
+                s, e = times[i]
+                s.record(stream)
+            if kern is not None:
+                G.gemm_profile_events(*kern[i])
+            c.launch()
+            if kern is not None:
+                G.gemm_profile_events(None, None)
+            if times is not None:
+                e.record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in cases] for _ in range(args.steps)]
+    kev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in cases] for _ in range(args.steps)]
+    for row in kev:  # materialise the event handles
+        for s, e in row:
+            s.record(stream)
+            e.record(stream)
+    torch.cuda.synchronize()
+
+    uuid = str(getattr(torch.cuda.get_device_properties(dev), "uuid", "") or "")
+    if uuid and not uuid.startswith("GPU-"):
+        uuid = "GPU-" + uuid
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    launches0 = G.gemm_launch_count()
+    t0 = time.perf_counter()
+    for k in range(args.steps):
+        step(ev[k], kev[k])
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    launches = G.gemm_launch_count() - launches0
+    if world > 1:
+        torch.distributed.barrier()
+    # the timed region is short: keep sampling clocks over the same work for
+    # about a second more so the clock record has samples under load
+    t1 = time.perf_counter()
+    while time.perf_counter() - t1 < 1.0:
+        step()
+    torch.cuda.synchronize()
+    sampler.stop()
+
+    per_gemm_ms = [[ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(args.steps)] for i in range(len(cases))]
+    per_kern_ms = [[kev[k][i][0].elapsed_time(kev[k][i][1]) for k in range(args.steps)] for i in range(len(cases))]
+    gemm_ms = sum(sum(x) for x in per_gemm_ms) / args.steps  # device ms per step
+    ops = sum(c.g.flops for c in cases)
+
+    # e2e: host buffers, copies inside the timed events
+    e2e_ms = None
+    if not args.no_e2e:
+        for _ in range(2):
+            for c in cases:
+                c.launch_e2e()
+        torch.cuda.synchronize()
+        e_ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 for _ in cases] for _ in range(args.steps)]
+        for k in range(args.steps):
+            for i, c in enumerate(cases):
+                flush.fill_(float(i))
+                e_ev[k][i][0].record(stream)
+                c.launch_e2e()
+                e_ev[k][i][1].record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = sum(e_ev[k][i][0].elapsed_time(e_ev[k][i][1]) for k in range(args.steps)
+                     for i in range(len(cases))) / args.steps
+
+    # max over ranks
+    vals = torch.tensor([gemm_ms, e2e_ms or 0.0, wall], dtype=torch.float64, device=dev)
+    if world > 1:
+        torch.distributed.all_reduce(vals, op=torch.distributed.ReduceOp.MAX)
+    gemm_ms, e2e_max, wall = vals.tolist()
+
+    peaks, peak_src = load_peaks()
+    bf16_peak = float(peaks.get("bf16_tflops", FALLBACK["bf16_tflops"]))
+    per = []
+    for i, c in enumerate(cases):
+        ms = statistics.median(per_gemm_ms[i])
+        kms = statistics.median(per_kern_ms[i])
+        tops = c.g.flops / (ms * 1e-3) / 1e12
+        per.append({"gemm": c.g.name, "ms": round(ms, 5), "tc_kernel_ms": round(kms, 5),
+                    "tops": round(tops, 2), "frac_of_bf16_peak": round(tops / bf16_peak, 4),
+                    "best_ms": round(min(per_gemm_ms[i]), 5)})
+    # dominant kernel: the tensor-core kernel of the GEMM with the largest time
+    dom = max(range(len(cases)), key=lambda i: statistics.mean(per_gemm_ms[i]))
+    dk_ms = statistics.mean(per_kern_ms[dom])
+    achieved = cases[dom].g.flops / (dk_ms * 1e-3) / 1e12
+    traffic = load_traffic(cases[dom].g.name)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, args.cpu_seconds)
+
+    value = world * ops / (gemm_ms * 1e-3) / 1e12
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": "TOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(gemm_ms, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int8->int32 and bf16->fp32->bf16", "data": "synthetic (seeded, workloads.py)",
+        "config": {"workload": wl.name, "description": wl.description,
+                   "gemms": [c.g.name for c in cases], "l2": "flushed (512 MiB write) before every timed GEMM",
+                   "parallelism": f"replicas x{world}"},
+        "per_gemm": per,
+        "roofline": {"bound": "tensor", "kernel": f"gemm_tc_kernel ({cases[dom].g.name})",
+                     "achieved": round(achieved, 2), "peak": bf16_peak, "unit": "TFLOP/s",
+                     "frac": round(achieved / bf16_peak, 4), "traffic": traffic,
+                     "peak_source": f"{peak_src} bf16 dense (burst)"},
+        "e2e": None if e2e_ms is None else {
+            "value": round(world * ops / (e2e_max * 1e-3) / 1e12, 3), "unit": "TOPS",
+            "h2d_bytes_per_step": sum(c.h2d for c in cases), "d2h_bytes_per_step": sum(c.d2h for c in cases)},
+        "gpu_launches": int(launches),
+        "wall_s_timed_region": round(wall, 4),
+        "clocks": sampler.summary(),
+        "cpu_baseline": cpu,
+    }
+    return line
+
+
+def load_traffic(name):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary (profiles/traffic.json), or None when not captured for it."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d.get(name)
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------ CPU oracle
+
+def _oracle_rows(g: W.Gemm, A, B, rows):
+    import oracle
+    As = np.ascontiguousarray(A[:rows])
+    if g.dtype == "int8":
+        oracle.gemm_s8(As, B, g.layout)
+    else:
+        oracle.gemm_bf16(As, B, g.layout)
+
+
+def cpu_baseline(wl, seconds):
+    """Oracle throughput on whole rows of C of every GEMM of the workload,
+    about `seconds` of CPU work in total."""
+    import oracle
+    oracle.build()
+    budget = seconds / len(wl.gemms)
+    ops = 0
+    t_total = 0.0
+    rows_used = []
+    for g in wl.gemms:
+        A, B = W.make_inputs(g)
+        t0 = time.perf_counter()
+        _oracle_rows(g, A, B, 1)
+        t1 = time.perf_counter() - t0
+        rows = max(1, min(g.M, int(budget / max(t1, 1e-6))))
+        t0 = time.perf_counter()
+        _oracle_rows(g, A, B, rows)
+        dt = time.perf_counter() - t0
+        ops += 2 * rows * g.N * g.K
+        t_total += dt
+        rows_used.append(f"{g.name}:{rows}rows")
+    return {"value": round(ops / t_total / 1e12, 6), "unit": "TOPS", "cores": oracle.num_threads(),
+            "kind": "oracle", "seconds": round(t_total, 2),
+            "sample": "whole rows of C per GEMM (" + ", ".join(rows_used) + ")"}
+
+
+def run_reference(args, rank, world):
+    """The oracle, as it stands, timed on this host's cores on bounded
+    samples (whole rows of C) of every GEMM of the workload."""
+    import oracle
+    oracle.build()
+    wl = W.WORKLOADS[args.workload]
+    inputs = [W.make_inputs(g) for g in wl.gemms]
+    per_step = args.cpu_seconds_per_step / len(wl.gemms)
+    rows = []
+    for g, (A, B) in zip(wl.gemms, inputs):
+        t0 = time.perf_counter()
+        _oracle_rows(g, A, B, 1)
+        t1 = time.perf_counter() - t0
+        rows.append(max(1, min(g.M, int(per_step / max(t1, 1e-6)))))
+    for _ in range(args.warmup):
+        for g, (A, B), r in zip(wl.gemms, inputs, rows):
+            _oracle_rows(g, A, B, max(1, r // 8))
+    ops, t_total = 0, 0.0
+    for _ in range(args.steps):
+        for g, (A, B), r in zip(wl.gemms, inputs, rows):
+            t0 = time.perf_counter()
+            _oracle_rows(g, A, B, r)
+            t_total += time.perf_counter() - t0
+            ops += 2 * r * g.N * g.K
+    value = ops / t_total / 1e12
+    sample = "whole rows of C per GEMM per step (" + ", ".join(
+        f"{g.name}:{r}rows" for g, r in zip(wl.gemms, rows)) + ")"
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t_total / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int8->int64 and bf16->f64 (oracle)", "data": "synthetic (seeded, workloads.py)",
+        "config": {"workload": wl.name, "description": wl.description, "gemms": [g.name for g in wl.gemms]},
+        "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": oracle.num_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="square_sweep_512_4096", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=16.0)
+    ap.add_argument("--cpu-seconds-per-step", type=float, default=6.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=dev)
+    line = run_ours(args, rank, world, dev)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,119 @@
+/*
+ * gb300_gemm.h -- C ABI of the GB300 (sm_103a) dense GEMM library.
+ *
+ * The operation (Sec. 4.1 of "Striking the Balance: GEMM Performance
+ * Optimization Across Generations of Ryzen AI NPUs", arXiv 2512.13282):
+ *
+ *     C = A . B,   A is M x K, B is K x N, C is M x N,
+ *
+ * with A and C row-major and B either row-major (K x N) or column-major
+ * (stored N x K, K contiguous) (Sec. 4.2.2).  Two precisions (Sec. 5.1,
+ * Table 1): "int8-int32" -- int8 operands, exact int32 result -- and
+ * "bf16-bf16" -- bf16 operands, float32 accumulation, bf16 result rounded to
+ * nearest, ties to even.  Arbitrary M, N, K are supported (Sec. 5.3.1 pads to
+ * the design's native size; here partial edge tiles are clipped instead, so
+ * nothing outside [0,M) x [0,N) of C is ever written).
+ *
+ * Conventions shared by every entry point:
+ *   - Pointers A, B, C are DEVICE pointers owned by the caller; the library
+ *     never frees them.  A, B and C must not overlap.
+ *   - Leading dimensions are in elements: row i of A starts at A + i*lda;
+ *     row k of a row-major B at B + k*ldb, row j of a column-major B (its
+ *     column j) at B + j*ldb; row i of C at C + i*ldc.
+ *   - The call is asynchronous on `stream` (0 = legacy default stream): it
+ *     validates, enqueues its kernels and returns without synchronising.
+ *   - M == 0 or N == 0 is a no-op returning GEMM_OK; K == 0 writes zeros.
+ *   - Errors are returned as status codes; nothing is thrown across the ABI.
+ *   - The library keeps a lazily grown device workspace (for operand staging
+ *     and split-K partials), allocated stream-ordered on first need and
+ *     released by gemm_release_resources().  Calls on different streams that
+ *     both need the workspace must be ordered by the caller.
+ */
+#ifndef GB300_GEMM_H
+#define GB300_GEMM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *gemm_stream_t; /* same object as cudaStream_t */
+
+typedef enum {
+  GEMM_OK = 0,
+  GEMM_ERR_INVALID_ARG = 1, /* negative size, null pointer with nonzero extent,
+                               lda < K, ldb < N (row-major) or < K (column-major),
+                               ldc < N, unknown layout flag */
+  GEMM_ERR_UNSUPPORTED = 2, /* int8 with K > 131071: 131072 * (-128)^2 = 2^31 no
+                               longer fits int32, so exactness is not possible;
+                               or a device that is not sm_103 */
+  GEMM_ERR_CUDA = 3,        /* a CUDA runtime/driver call or launch failed */
+  GEMM_ERR_TIMEOUT = 4      /* a bounded on-device wait expired; reported by
+                               gemm_device_status() after the stream is synced */
+} gemm_status_t;
+
+typedef enum {
+  GEMM_B_ROW_MAJOR_KxN = 0, /* B(k, n) = B[k*ldb + n] */
+  GEMM_B_COL_MAJOR_NxK = 1  /* B(k, n) = B[n*ldb + k] */
+} gemm_b_layout_t;
+
+/*
+ * int8-int32 (Sec. 5.1, Table 1): C[i][j] = sum_k A[i][k] * B(k, j), exact.
+ *   A: int8, M x K row-major (lda >= K).  B: int8, layout per b_layout.
+ *   C: int32, M x N row-major (ldc >= N), fully overwritten in [0,M) x [0,N).
+ *   K <= 131071 guarantees the exact sum fits int32; larger K returns
+ *   GEMM_ERR_UNSUPPORTED.
+ */
+gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K,
+                            const int8_t *A, int64_t lda,
+                            const int8_t *B, int64_t ldb, int b_layout,
+                            int32_t *C, int64_t ldc, gemm_stream_t stream);
+
+/*
+ * bf16-bf16 (Sec. 5.1, Table 1): C[i][j] = rne_bf16(sum_k a_ik * b_kj) with
+ * the sum accumulated in float32 (any order) and rounded once to bf16,
+ * nearest-even.  A, B, C are bf16 bit patterns (uint16_t).
+ *   A: M x K row-major (lda >= K).  B: layout per b_layout.
+ *   C: M x N row-major (ldc >= N), fully overwritten in [0,M) x [0,N).
+ * Accuracy contract: |C - ref| <= 2^-8 |ref| + 2^-20 sum_k |a_ik b_kj| per
+ * element, ref being the exact sum.
+ */
+gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K,
+                                    const uint16_t *A, int64_t lda,
+                                    const uint16_t *B, int64_t ldb, int b_layout,
+                                    uint16_t *C, int64_t ldc, gemm_stream_t stream);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *gemm_status_string(gemm_status_t status);
+
+/*
+ * Reads and clears the device error word that kernels set when a bounded
+ * wait expires (GEMM_ERR_TIMEOUT) on the current device.  Synchronises the
+ * device first.  Returns GEMM_OK if no kernel reported an error.
+ */
+gemm_status_t gemm_device_status(void);
+
+/* Frees the workspace and cached state of the current device.  The caller
+ * must ensure no library kernel is still running. */
+void gemm_release_resources(void);
+
+/* Number of kernel launches the library has enqueued since load (all
+ * devices); lets a caller count the kernels a region of work launched. */
+uint64_t gemm_launch_count(void);
+
+/*
+ * Profiling aid.  With both arguments non-NULL (cudaEvent_t handles created
+ * by the caller), every following GEMM call records `start_event` on its
+ * stream just before launching its tensor-core kernel and `stop_event` just
+ * after, so the time between them covers that kernel alone -- not the
+ * operand staging or the split-K reduction passes.  Pass NULL, NULL to stop.
+ * Process-wide setting; not meant for concurrent callers.
+ */
+void gemm_profile_events(void *start_event, void *stop_event);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GB300_GEMM_H */

@@ -1,0 +1,357 @@
+// gemm_api.cu -- the C ABI (include/gb300_gemm.h): argument checks, tile
+// and split-K selection, operand staging, TMA descriptor encoding, launches.
+//
+// One compiled design serves every problem size: as in the paper
+// (Sec. 5.3.1), only the tile counts and the number of K steps change from
+// one GEMM to the next, and those are runtime kernel arguments here.
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "gb300_gemm.h"
+#include "gemm_internal.h"
+
+using namespace gb300;
+
+// Device error word: kernels record kDevErrTimeout here when a bounded wait
+// expires.  Read and cleared by gemm_device_status().
+__device__ uint32_t g_gemm_dev_err = 0;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+constexpr int64_t kMaxExactK = 131071;  // 131072 * 2^14 = 2^31 overflows int32
+
+struct DeviceState {
+  bool ready = false;
+  int sms = 0;
+  uint32_t *err = nullptr;
+  void *ws = nullptr;
+  size_t ws_bytes = 0;
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::atomic<uint64_t> g_launches{0};
+cudaEvent_t g_prof_start = nullptr, g_prof_stop = nullptr;
+
+uint64_t wait_limit_ns() {
+  static uint64_t v = [] {
+    const char *s = std::getenv("GB300_GEMM_WAIT_LIMIT_MS");
+    const double ms = s ? std::atof(s) : 2000.0;
+    return (uint64_t)((ms > 0 ? ms : 2000.0) * 1e6);
+  }();
+  return v;
+}
+
+gemm_status_t device_state(DeviceState **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return GEMM_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceState &d = g_dev[dev];
+  if (!d.ready) {
+    int major = 0, minor = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return GEMM_ERR_CUDA;
+    if (major != 10 || minor != 3) return GEMM_ERR_UNSUPPORTED;  // built for sm_103a only
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&d.err), g_gemm_dev_err) != cudaSuccess)
+      return GEMM_ERR_CUDA;
+    if (!g_encode) {
+      cudaDriverEntryPointQueryResult q;
+      void *fn = nullptr;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || !fn)
+        return GEMM_ERR_CUDA;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    d.sms = sms;
+    d.ready = true;
+  }
+  *out = &d;
+  return GEMM_OK;
+}
+
+// Grow the device workspace (stream-ordered) to at least `bytes`.
+gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
+  if (bytes <= d.ws_bytes) return GEMM_OK;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (bytes <= d.ws_bytes) return GEMM_OK;
+  if (d.ws) {
+    if (cudaFreeAsync(d.ws, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    d.ws = nullptr;
+    d.ws_bytes = 0;
+  }
+  const size_t grown = bytes + bytes / 4;
+  if (cudaMallocAsync(&d.ws, grown, st) != cudaSuccess) {
+    d.ws = nullptr;
+    return GEMM_ERR_CUDA;
+  }
+  d.ws_bytes = grown;
+  return GEMM_OK;
+}
+
+// Test and benchmark overrides of the planner: GB300_GEMM_BN (128 or 256)
+// forces the tile width, GB300_GEMM_SPLITS (>= 1) the split-K factor.
+int env_int(const char *name) {
+  const char *s = std::getenv(name);
+  return s ? std::atoi(s) : 0;
+}
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// 2-D bf16 tensor map: inner extent `inner` (contiguous), outer extent
+// `outer`, row pitch `ld` elements, box box_inner x box_outer, 128-byte
+// swizzle.  Out-of-range box elements read as zero.
+bool encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t ld,
+                    uint32_t box_inner, uint32_t box_outer) {
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {ld * 2};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+gemm_status_t check_common(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,
+                           int64_t ldb, int layout, const void *C, int64_t ldc) {
+  if (M < 0 || N < 0 || K < 0) return GEMM_ERR_INVALID_ARG;
+  if (layout != GEMM_B_ROW_MAJOR_KxN && layout != GEMM_B_COL_MAJOR_NxK) return GEMM_ERR_INVALID_ARG;
+  if (M == 0 || N == 0) return GEMM_OK;
+  if (!C || ldc < N) return GEMM_ERR_INVALID_ARG;
+  if (K > 0) {
+    if (!A || !B || lda < K) return GEMM_ERR_INVALID_ARG;
+    if (layout == GEMM_B_ROW_MAJOR_KxN ? ldb < N : ldb < K) return GEMM_ERR_INVALID_ARG;
+  }
+  // Index arithmetic inside the kernels uses int for tile and K-block
+  // counters and TMA coordinates: keep every extent below 2^31.
+  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return GEMM_ERR_UNSUPPORTED;
+  return GEMM_OK;
+}
+
+struct Plan {
+  TcVariant v;
+  TcParams p;
+  int grid;
+};
+
+// Tile width, split-K factor and grid for an M x N x K problem on `sms` SMs.
+// BN = 256 when that still yields a full wave of tiles, else 128.  Split K
+// only when the tile count leaves most SMs idle, keeping >= 4 k-blocks per
+// split; the reduction then runs as a separate pass over fp32/int32 partials.
+Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms) {
+  Plan pl{};
+  const int64_t tiles_m = ceil_div(M, kBM);
+  int bn = (N > 128 && tiles_m * ceil_div(N, 256) >= sms) ? 256 : 128;
+  const int force_bn = env_int("GB300_GEMM_BN");
+  if (force_bn == 128 || force_bn == 256) bn = force_bn;
+  const int64_t tiles_n = ceil_div(N, bn);
+  const int64_t tiles = tiles_m * tiles_n;
+  const int64_t num_kb = ceil_div(K, kBK);
+  int64_t splits = 1;
+  if (tiles * 2 <= sms && num_kb >= 8) {
+    splits = sms / tiles;
+    if (splits > num_kb / 4) splits = num_kb / 4;
+    if (splits > 16) splits = 16;
+    if (splits < 1) splits = 1;
+  }
+  const int force_splits = env_int("GB300_GEMM_SPLITS");
+  if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
+  const int64_t kb_per = ceil_div(num_kb, splits);
+  splits = ceil_div(num_kb, kb_per);
+  pl.v = TcVariant{bn, b_kmajor, epi};
+  TcParams &p = pl.p;
+  p.M = (int)M;
+  p.N = (int)N;
+  p.K = (int)K;
+  p.tiles_m = (int)tiles_m;
+  p.tiles_n = (int)tiles_n;
+  p.num_kb = (int)num_kb;
+  p.splits = (int)splits;
+  p.kb_per_split = (int)kb_per;
+  p.slab_kb = epi == kEpiS32 ? 1024 / kBK : (int)num_kb;
+  p.group_m = 8;
+  const int64_t units = tiles * splits;
+  pl.grid = (int)(units < sms ? units : sms);
+  return pl;
+}
+
+struct WsLayout {
+  size_t a_off = 0, b_off = 0, part_off = 0, total = 0;
+};
+
+// Shared path after staging: encode maps, launch the tcgen05 kernel and the
+// split-K reduction.
+gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, const uint16_t *B,
+                     int64_t ldb, void *C, int64_t ldc, int esize, void *partials, cudaStream_t st) {
+  TcParams &p = pl.p;
+  CUtensorMap ta, tb;
+  if (!encode_bf16_2d(&ta, A, (uint64_t)p.K, (uint64_t)p.M, (uint64_t)lda, kBK, kBM)) return GEMM_ERR_CUDA;
+  const bool ok_b = pl.v.b_kmajor
+                        ? encode_bf16_2d(&tb, B, (uint64_t)p.K, (uint64_t)p.N, (uint64_t)ldb, kBK, pl.v.bn)
+                        : encode_bf16_2d(&tb, B, (uint64_t)p.N, (uint64_t)p.K, (uint64_t)ldb, 64, kBK);
+  if (!ok_b) return GEMM_ERR_CUDA;
+  p.C = C;
+  p.ldc = ldc;
+  p.c_vec = aligned16(C) && ((ldc * esize) % 16 == 0);
+  p.ws = partials;
+  p.err = d.err;
+  p.wait_limit_ns = wait_limit_ns();
+  const bool prof = g_prof_start && g_prof_stop;
+  if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  cudaError_t e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, p, pl.grid, st)
+                                      : launch_tc_bf16(pl.v, ta, tb, p, pl.grid, st);
+  g_launches.fetch_add(1);
+  if (e != cudaSuccess) return GEMM_ERR_CUDA;
+  if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (p.splits > 1) {
+    e = pl.v.epi == kEpiS32
+            ? launch_splitk_reduce_s32(static_cast<const int32_t *>(partials), p.splits, p.M, p.N,
+                                       static_cast<int32_t *>(C), ldc, d.sms, st)
+            : launch_splitk_reduce_bf16(static_cast<const float *>(partials), p.splits, p.M, p.N,
+                                        static_cast<uint16_t *>(C), ldc, d.sms, st);
+    g_launches.fetch_add(1);
+    if (e != cudaSuccess) return GEMM_ERR_CUDA;
+  }
+  return GEMM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint16_t *A, int64_t lda,
+                                    const uint16_t *B, int64_t ldb, int b_layout, uint16_t *C,
+                                    int64_t ldc, gemm_stream_t stream) {
+  gemm_status_t s = check_common(M, N, K, A, lda, B, ldb, b_layout, C, ldc);
+  if (s != GEMM_OK || M == 0 || N == 0) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  DeviceState *d = nullptr;
+  if ((s = device_state(&d)) != GEMM_OK) return s;
+  if (K == 0) {
+    g_launches.fetch_add(1);
+    return launch_zero_fill(C, M, N, ldc, 2, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+  }
+  const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
+  Plan pl = make_plan(M, N, K, b_kmajor, kEpiBf16, d->sms);
+  // TMA needs 16-byte aligned bases and row pitches; re-pitch an operand
+  // that is not, into the workspace.
+  const bool pack_a = !(aligned16(A) && (lda * 2) % 16 == 0);
+  const bool pack_b = !(aligned16(B) && (ldb * 2) % 16 == 0);
+  const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
+  const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;
+  WsLayout L;
+  size_t off = 0;
+  if (pack_a) { L.a_off = off; off = align_up(off + (size_t)M * lda_p * 2, 256); }
+  if (pack_b) { L.b_off = off; off = align_up(off + (size_t)b_rows * ldb_p * 2, 256); }
+  if (pl.p.splits > 1) { L.part_off = off; off = align_up(off + (size_t)pl.p.splits * M * N * 4, 256); }
+  L.total = off;
+  if (L.total && (s = ensure_workspace(*d, L.total, st)) != GEMM_OK) return s;
+  uint8_t *ws = static_cast<uint8_t *>(d->ws);
+  const uint16_t *Au = A, *Bu = B;
+  int64_t lda_u = lda, ldb_u = ldb;
+  if (pack_a) {
+    uint16_t *dst = reinterpret_cast<uint16_t *>(ws + L.a_off);
+    g_launches.fetch_add(1);
+    if (launch_pack_u16(A, M, K, lda, dst, lda_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    Au = dst;
+    lda_u = lda_p;
+  }
+  if (pack_b) {
+    uint16_t *dst = reinterpret_cast<uint16_t *>(ws + L.b_off);
+    g_launches.fetch_add(1);
+    if (launch_pack_u16(B, b_rows, b_cols, ldb, dst, ldb_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    Bu = dst;
+    ldb_u = ldb_p;
+  }
+  return run_tc(*d, pl, Au, lda_u, Bu, ldb_u, C, ldc, 2, pl.p.splits > 1 ? ws + L.part_off : nullptr, st);
+}
+
+gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
+                            const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
+                            gemm_stream_t stream) {
+  gemm_status_t s = check_common(M, N, K, A, lda, B, ldb, b_layout, C, ldc);
+  if (s != GEMM_OK || M == 0 || N == 0) return s;
+  if (K > kMaxExactK) return GEMM_ERR_UNSUPPORTED;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  DeviceState *d = nullptr;
+  if ((s = device_state(&d)) != GEMM_OK) return s;
+  if (K == 0) {
+    g_launches.fetch_add(1);
+    return launch_zero_fill(C, M, N, ldc, 4, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+  }
+  const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
+  Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
+  // Stage both operands as bf16 (exact for int8) with 16-byte aligned rows.
+  const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
+  const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;
+  WsLayout L;
+  size_t off = 0;
+  L.a_off = off;
+  off = align_up(off + (size_t)M * lda_p * 2, 256);
+  L.b_off = off;
+  off = align_up(off + (size_t)b_rows * ldb_p * 2, 256);
+  if (pl.p.splits > 1) { L.part_off = off; off = align_up(off + (size_t)pl.p.splits * M * N * 4, 256); }
+  L.total = off;
+  if ((s = ensure_workspace(*d, L.total, st)) != GEMM_OK) return s;
+  uint8_t *ws = static_cast<uint8_t *>(d->ws);
+  uint16_t *Ab = reinterpret_cast<uint16_t *>(ws + L.a_off);
+  uint16_t *Bb = reinterpret_cast<uint16_t *>(ws + L.b_off);
+  g_launches.fetch_add(2);
+  if (launch_s8_to_bf16(A, M, K, lda, Ab, lda_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (launch_s8_to_bf16(B, b_rows, b_cols, ldb, Bb, ldb_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, pl.p.splits > 1 ? ws + L.part_off : nullptr, st);
+}
+
+const char *gemm_status_string(gemm_status_t status) {
+  switch (status) {
+    case GEMM_OK: return "GEMM_OK";
+    case GEMM_ERR_INVALID_ARG: return "GEMM_ERR_INVALID_ARG: invalid argument";
+    case GEMM_ERR_UNSUPPORTED: return "GEMM_ERR_UNSUPPORTED: unsupported size or device";
+    case GEMM_ERR_CUDA: return "GEMM_ERR_CUDA: CUDA call or launch failed";
+    case GEMM_ERR_TIMEOUT: return "GEMM_ERR_TIMEOUT: a bounded device wait expired";
+  }
+  return "unknown gemm_status_t";
+}
+
+gemm_status_t gemm_device_status(void) {
+  DeviceState *d = nullptr;
+  gemm_status_t s = device_state(&d);
+  if (s != GEMM_OK) return s;
+  if (cudaDeviceSynchronize() != cudaSuccess) return GEMM_ERR_CUDA;
+  uint32_t v = 0;
+  if (cudaMemcpy(&v, d->err, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (v != 0) {
+    const uint32_t zero = 0;
+    if (cudaMemcpy(d->err, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return GEMM_ERR_CUDA;
+  }
+  return v == 0 ? GEMM_OK : static_cast<gemm_status_t>(v);
+}
+
+void gemm_release_resources(void) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceState &d = g_dev[dev];
+  if (d.ws) cudaFree(d.ws);
+  d.ws = nullptr;
+  d.ws_bytes = 0;
+}
+
+uint64_t gemm_launch_count(void) { return g_launches.load(); }
+
+void gemm_profile_events(void *start_event, void *stop_event) {
+  g_prof_start = static_cast<cudaEvent_t>(start_event);
+  g_prof_stop = static_cast<cudaEvent_t>(stop_event);
+}
+
+}  // extern "C"

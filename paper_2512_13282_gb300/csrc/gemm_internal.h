@@ -1,0 +1,47 @@
+// gemm_internal.h -- host-side declarations shared by the library's
+// translation units (not part of the public ABI).
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "gemm_tc.cuh"
+
+namespace gb300 {
+
+// One compiled variant of the tcgen05 kernel.
+struct TcVariant {
+  int bn;        // 128 or 256
+  bool b_kmajor; // B stored N x K (K contiguous)
+  int epi;       // kEpiBf16 or kEpiS32
+};
+
+// Shared-memory bytes and threads of a variant (for occupancy/launch).
+int tc_smem_bytes(const TcVariant &v);
+int tc_threads(const TcVariant &v);
+
+// Launch the persistent tcgen05 GEMM kernel (gemm_tc_bf16.cu / gemm_tc_s32.cu).
+cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
+                           const TcParams &p, int grid, cudaStream_t st);
+cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
+                          const TcParams &p, int grid, cudaStream_t st);
+
+// Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
+// int8 -> bf16 (exact), rows x cols, arbitrary source leading dimension.
+cudaError_t launch_s8_to_bf16(const int8_t *src, int64_t rows, int64_t cols, int64_t ld_src,
+                              uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st);
+// bf16 copy into an aligned buffer (re-pitching a misaligned operand).
+cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int64_t ld_src,
+                            uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st);
+// Fill an M x N block of 16- or 32-bit elements with zero.
+cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esize, int sms,
+                             cudaStream_t st);
+// Split-K reduction: C = round(sum over splits of ws[s]) (fp32 -> bf16 RNE)
+// or C = sum of int32 partials.
+cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, int64_t N,
+                                      uint16_t *C, int64_t ldc, int sms, cudaStream_t st);
+cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N,
+                                     int32_t *C, int64_t ldc, int sms, cudaStream_t st);
+
+}  // namespace gb300

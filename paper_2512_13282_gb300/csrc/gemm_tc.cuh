@@ -1,0 +1,357 @@
+// gemm_tc.cuh -- persistent, warp-specialised tcgen05 GEMM kernel.
+//
+// One CTA per SM loops over output tiles (the paper's output-stationary
+// mapping, Sec. 4.2.1: M and N are spread in space over independent workers,
+// K is reduced in time into a stationary accumulator).  Roles:
+//   warp 0 (one lane)  TMA producer: streams 128 x 64 A boxes and BN x 64 B
+//                      boxes into a STAGES-deep shared-memory ring (the
+//                      paper's double-buffered L1/L2 input tiles, Sec. 4.2.1,
+//                      deepened), each stage guarded by a full/empty mbarrier
+//                      pair.  The box shapes and the 128-byte swizzle play the
+//                      part of the paper's on-the-fly DMA layout transforms
+//                      (Sec. 4.3): matrices stay row-/column-major in memory.
+//   warp 1 (one lane)  MMA issuer: tcgen05.mma kind::f16 (bf16 x bf16 -> fp32)
+//                      into one of two TMEM accumulators; the first MMA of a
+//                      tile overwrites instead of accumulating, which takes
+//                      the place of the paper's zeroing kernel (Sec. 4.2.1).
+//   warps 2..          epilogue: TMEM -> registers -> bf16 (RNE) or int32 ->
+//                      global memory, masked at the M/N edges.  Two
+//                      accumulators let the epilogue of one tile overlap the
+//                      main loop of the next (the paper keeps a single C
+//                      buffer for lack of L1 space, Sec. 5.3.2; TMEM has room
+//                      for two).
+//
+// Exact int8 emulation (kEpiS32): int8 operands, staged as bf16 (every int8
+// value is exact in bf16), are multiplied on the bf16 pipe.  A product is at
+// most 2^14 in magnitude, so any partial sum of at most 1024 of them is an
+// integer of magnitude <= 2^24 and exact in fp32.  The MMA warp therefore
+// closes the accumulator every `slab_kb` k-blocks (slab_kb * 64 <= 1024 K
+// elements); the epilogue converts each slab's fp32 sums to int32 (exactly)
+// and adds them in int32 registers.  The final int32 is exact whenever the
+// true result fits int32.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+#include "ptx.cuh"
+
+namespace gb300 {
+
+constexpr int kBM = 128;                    // MMA M (rows of C per tile)
+constexpr int kBK = 64;                     // K per stage: 64 bf16 = 128 bytes
+constexpr uint32_t kRowBytes = kBK * 2;     // one 128-byte swizzle row
+constexpr uint32_t kABytes = kBM * kRowBytes;
+
+enum EpiKind : int { kEpiBf16 = 0, kEpiS32 = 1 };
+
+struct TcParams {
+  int M, N, K;
+  int tiles_m, tiles_n;
+  int num_kb;        // ceil(K / kBK)
+  int splits;        // split-K factor (1: none)
+  int kb_per_split;  // k-blocks per split
+  int slab_kb;       // k-blocks per accumulator slab (>= kb_per_split for bf16)
+  int group_m;       // tiles of M per rasterisation group
+  void *C;           // bf16 or int32 output, row-major, leading dimension ldc
+  int64_t ldc;
+  int c_vec;         // C rows 16-byte aligned: vector stores allowed
+  void *ws;          // split-K partials, splits x M x N 32-bit words (fp32 or int32)
+  uint32_t *err;     // device error word
+  uint64_t wait_limit_ns;
+};
+
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
+struct TcCfg {
+  static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256, a multiple of 64");
+  static_assert(EPI_WARPS == 4 || EPI_WARPS == 8, "epilogue is one or two warpgroups");
+  static constexpr uint32_t kBBytes = BN * kRowBytes;
+  static constexpr uint32_t kStageBytes = kABytes + kBBytes;
+  static constexpr uint32_t kTmemCols = 2 * BN;  // two fp32 accumulators
+  static constexpr int kThreads = (2 + EPI_WARPS) * 32;
+  static constexpr int kColsPerThread = BN / (EPI_WARPS / 4);
+  static constexpr uint32_t kBarOffset = STAGES * kStageBytes;
+  static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
+  static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
+  static_assert(kTmemCols == 256 || kTmemCols == 512 || kTmemCols == 128, "TMEM columns");
+};
+
+struct Unit {
+  int tm, tn, split, kb0, kb1;
+};
+
+// Work unit u -> (tile, split).  Tiles are visited in groups of group_m
+// M-tiles so that CTAs running at the same time share A rows and B columns
+// in L2.
+__device__ __forceinline__ Unit decode_unit(const TcParams &p, int u) {
+  const int num_tiles = p.tiles_m * p.tiles_n;
+  Unit w;
+  w.split = u / num_tiles;
+  const int t = u - w.split * num_tiles;
+  const int group = p.group_m * p.tiles_n;
+  const int gid = t / group;
+  const int first_m = gid * p.group_m;
+  const int gm = min(p.tiles_m - first_m, p.group_m);
+  const int local = t - gid * group;
+  w.tm = first_m + local % gm;
+  w.tn = local / gm;
+  w.kb0 = w.split * p.kb_per_split;
+  w.kb1 = min(p.num_kb, w.kb0 + p.kb_per_split);
+  return w;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // round to nearest even
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// Store 32 consecutive 32-bit words of one row (fp32 partials or int32).
+__device__ __forceinline__ void store_row32(uint32_t *dst, int col, int N, bool vec,
+                                            const uint32_t (&v)[32]) {
+  if (vec && col + 32 <= N) {
+    uint4 *d = reinterpret_cast<uint4 *>(dst + col);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) d[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (col + i < N) dst[col + i] = v[i];
+  }
+}
+
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
+__global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const TcParams p) {
+  using Cfg = TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-byte alignment
+  uint8_t *base_ptr = smem_raw + (base - raw);
+  const uint32_t sA = base;
+  const uint32_t sB = base + STAGES * kABytes;
+  const uint32_t bars = base + Cfg::kBarOffset;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(base_ptr + Cfg::kBarOffset + Cfg::kNumBars * 8);
+  volatile uint32_t *abort_flag = tmem_slot + 1;
+
+  auto full_bar = [&](uint32_t s) { return bars + 8u * s; };
+  auto empty_bar = [&](uint32_t s) { return bars + 8u * (STAGES + s); };
+  auto accf_bar = [&](uint32_t b) { return bars + 8u * (2 * STAGES + b); };
+  auto acce_bar = [&](uint32_t b) { return bars + 8u * (2 * STAGES + 2 + b); };
+  const uint32_t drain_bar = bars + 8u * (2 * STAGES + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accf_bar(b), 1);
+      mbar_init(acce_bar(b), EPI_WARPS * 32);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0u;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) tmem_alloc<Cfg::kTmemCols>(smem_addr(tmem_slot));
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int num_units = p.tiles_m * p.tiles_n * p.splits;
+  constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint32_t g = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
+        const Unit w = decode_unit(p, u);
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+          const uint32_t s = g % STAGES, ph = (g / STAGES) & 1u;
+          if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, p.err, p.wait_limit_ns)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full_bar(s), Cfg::kStageBytes);
+          tma_load_2d(sA + s * kABytes, &tmA, kb * kBK, w.tm * kBM, full_bar(s));
+          const uint32_t b_dst = sB + s * Cfg::kBBytes;
+          if constexpr (B_KMAJOR) {
+            tma_load_2d(b_dst, &tmB, kb * kBK, w.tn * BN, full_bar(s));
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j)
+              tma_load_2d(b_dst + j * (kBK * 128), &tmB, w.tn * BN + 64 * j, kb * kBK, full_bar(s));
+          }
+          ++g;
+        }
+      }
+      // Every load this thread issued has landed before the CTA may exit.
+      const uint32_t first = g > (uint32_t)STAGES ? g - STAGES : 0u;
+      for (uint32_t i = first; i < g; ++i) mbar_wait_drain(full_bar(i % STAGES), (i / STAGES) & 1u, kDrainNs);
+    }
+    __syncwarp();  // lanes 1..31 wait here, so the warp reaches the CTA barrier converged
+  } else if (warp == 1) {
+    // ------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(kBM, BN, !B_KMAJOR);
+      uint32_t g = 0, acc_cnt = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
+        const Unit w = decode_unit(p, u);
+        for (int kb_s = w.kb0; ok && kb_s < w.kb1; kb_s += p.slab_kb) {
+          const int kb_e = min(w.kb1, kb_s + p.slab_kb);
+          const uint32_t b = acc_cnt & 1u, aph = (acc_cnt >> 1) & 1u;
+          if (!mbar_wait(acce_bar(b), aph ^ 1u, abort_flag, p.err, p.wait_limit_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+          const uint32_t d_tmem = tmem_base + b * BN;
+          for (int kb = kb_s; kb < kb_e; ++kb) {
+            const uint32_t s = g % STAGES, ph = (g / STAGES) & 1u;
+            if (!mbar_wait(full_bar(s), ph, abort_flag, p.err, p.wait_limit_ns)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after_sync();
+            const uint32_t a0 = sA + s * kABytes;
+            const uint32_t b0 = sB + s * Cfg::kBBytes;
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              // K-major, 128-byte swizzle: rows 128 B apart, 8-row atoms
+              // 1024 B apart; one MMA step of K = 16 is 32 bytes along a row.
+              const uint64_t ad = smem_desc_sw128(a0 + k * 32, 16, 1024);
+              // MN-major B: 64-wide N chunks kBK*128 B apart (LBO), 8-row
+              // K groups 1024 B apart (SBO); a K step of 16 rows is 2048 B.
+              const uint64_t bd = B_KMAJOR ? smem_desc_sw128(b0 + k * 32, 16, 1024)
+                                           : smem_desc_sw128(b0 + k * 2048, kBK * 128, 1024);
+              tc_mma_bf16(d_tmem, ad, bd, idesc, (kb > kb_s || k > 0) ? 1u : 0u);
+            }
+            tc_commit(empty_bar(s));  // stage s is free once these MMAs finish
+            ++g;
+          }
+          if (!ok) break;
+          tc_commit(accf_bar(b));  // accumulator b is ready for the epilogue
+          ++acc_cnt;
+        }
+      }
+      // All MMAs complete before TMEM is released.
+      tc_commit(drain_bar);
+      mbar_wait_drain(drain_bar, 0, kDrainNs);
+    }
+    __syncwarp();
+  } else {
+    // --------------------------------------------------------- epilogue
+    constexpr int CPT = Cfg::kColsPerThread;
+    const int ew = warp - 2;
+    const int quad = warp & 3;  // a warp may only touch TMEM lanes 32*(warp%4) ..
+    const int colpart = ew >> 2;
+    const int row_in_tile = quad * 32 + lane;
+    const bool split = p.splits > 1;
+    const bool ws_vec = (p.N & 3) == 0;
+    uint32_t acc_cnt = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
+      const Unit w = decode_unit(p, u);
+      const int64_t row = (int64_t)w.tm * kBM + row_in_tile;
+      const bool row_ok = row < p.M;
+      const int col0 = w.tn * BN + colpart * CPT;
+      if constexpr (EPI == kEpiS32) {
+        int32_t acc[CPT];
+#pragma unroll
+        for (int i = 0; i < CPT; ++i) acc[i] = 0;
+        for (int kb_s = w.kb0; kb_s < w.kb1; kb_s += p.slab_kb) {
+          const uint32_t b = acc_cnt & 1u, aph = (acc_cnt >> 1) & 1u;
+          // all lanes agree (and reconverge) before the warp-wide TMEM loads
+          if (!__all_sync(0xffffffffu, mbar_wait(accf_bar(b), aph, abort_flag, p.err, p.wait_limit_ns))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+          const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
+#pragma unroll
+          for (int c = 0; c < CPT / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld_32x32b_x32(t0 + c * 32, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) acc[c * 32 + i] += __float2int_rn(__uint_as_float(r[i]));
+          }
+          tc_fence_before_sync();
+          mbar_arrive(acce_bar(b));
+          ++acc_cnt;
+        }
+        if (!ok) break;
+        if (row_ok) {
+          uint32_t *dst = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                                : reinterpret_cast<uint32_t *>(p.C) + row * p.ldc;
+          const bool vec = split ? ws_vec : (p.c_vec != 0);
+#pragma unroll
+          for (int c = 0; c < CPT / 32; ++c) {
+            uint32_t v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
+            store_row32(dst, col0 + c * 32, p.N, vec, v);
+          }
+        }
+      } else {
+        const uint32_t b = acc_cnt & 1u, aph = (acc_cnt >> 1) & 1u;
+        if (!__all_sync(0xffffffffu, mbar_wait(accf_bar(b), aph, abort_flag, p.err, p.wait_limit_ns))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
+#pragma unroll 1
+        for (int c = 0; c < CPT / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(t0 + c * 32, r);
+          tmem_ld_wait();
+          if (!row_ok) continue;
+          const int col = col0 + c * 32;
+          if (split) {
+            uint32_t *dst = reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N;
+            store_row32(dst, col, p.N, ws_vec, r);
+          } else {
+            uint16_t *dst = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
+            uint32_t h[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) h[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+            if (p.c_vec && col + 32 <= p.N) {
+              uint4 *d = reinterpret_cast<uint4 *>(dst + col);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) d[i] = make_uint4(h[4 * i], h[4 * i + 1], h[4 * i + 2], h[4 * i + 3]);
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (col + i < p.N) dst[col + i] = static_cast<uint16_t>(h[i >> 1] >> (16 * (i & 1)));
+            }
+          }
+        }
+        tc_fence_before_sync();
+        mbar_arrive(acce_bar(b));
+        ++acc_cnt;
+      }
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after_sync();
+    tmem_dealloc<Cfg::kTmemCols>(tmem_base);
+  }
+}
+
+}  // namespace gb300

@@ -1,0 +1,125 @@
+"""ctypes binding of the C ABI in ``include/gb300_gemm.h`` -- argument
+marshalling only; every step of the GEMM runs in the library's CUDA kernels.
+
+The functions keep the C names.  Pointer arguments accept either an integer
+device address or a CUDA ``torch.Tensor`` (its ``data_ptr()``); ``stream``
+accepts an integer ``cudaStream_t``, a ``torch.cuda.Stream`` or ``None``
+(torch's current stream on the current device).
+
+The library must have been built (``paper_2512_13282_gb300.build.build()``);
+there is no fallback: loading fails loudly if it is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from .build import LIB_PATH
+
+GEMM_OK = 0
+GEMM_ERR_INVALID_ARG = 1
+GEMM_ERR_UNSUPPORTED = 2
+GEMM_ERR_CUDA = 3
+GEMM_ERR_TIMEOUT = 4
+
+GEMM_B_ROW_MAJOR_KxN = 0
+GEMM_B_COL_MAJOR_NxK = 1
+
+_lock = threading.Lock()
+_lib = None
+
+
+class GemmError(RuntimeError):
+    def __init__(self, status: int):
+        self.status = int(status)
+        super().__init__(gemm_status_string(status))
+
+
+def library():
+    """The loaded ``libgb300gemm.so`` (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "paper_2512_13282_gb300.build.build() (no CPU fallback exists)")
+        lib = ctypes.CDLL(LIB_PATH)
+        i64, vp, ci = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int
+        for name in ("gemm_s8s8_s32", "gemm_bf16_f32acc_bf16"):
+            f = getattr(lib, name)
+            f.argtypes = [i64, i64, i64, vp, i64, vp, i64, ci, vp, i64, vp]
+            f.restype = ci
+        lib.gemm_status_string.argtypes = [ci]
+        lib.gemm_status_string.restype = ctypes.c_char_p
+        lib.gemm_device_status.argtypes = []
+        lib.gemm_device_status.restype = ci
+        lib.gemm_release_resources.argtypes = []
+        lib.gemm_release_resources.restype = None
+        lib.gemm_launch_count.argtypes = []
+        lib.gemm_launch_count.restype = ctypes.c_uint64
+        lib.gemm_profile_events.argtypes = [vp, vp]
+        lib.gemm_profile_events.restype = None
+        _lib = lib
+        return lib
+
+
+def _ptr(x) -> int:
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _stream(s) -> int:
+    if s is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream)
+    if isinstance(s, int):
+        return s
+    return int(s.cuda_stream)
+
+
+def gemm_s8s8_s32(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int:
+    """C (int32, M x N) = A (int8, M x K) . B (int8, K x N), exact."""
+    return int(library().gemm_s8s8_s32(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
+                                       _ptr(C), ldc, _stream(stream)))
+
+
+def gemm_bf16_f32acc_bf16(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int:
+    """C (bf16, M x N) = rne_bf16(A (bf16) . B (bf16)) with fp32 accumulation."""
+    return int(library().gemm_bf16_f32acc_bf16(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
+                                               _ptr(C), ldc, _stream(stream)))
+
+
+def gemm_status_string(status: int) -> str:
+    return library().gemm_status_string(int(status)).decode()
+
+
+def gemm_device_status() -> int:
+    return int(library().gemm_device_status())
+
+
+def gemm_release_resources() -> None:
+    library().gemm_release_resources()
+
+
+def gemm_launch_count() -> int:
+    return int(library().gemm_launch_count())
+
+
+def gemm_profile_events(start_event, stop_event) -> None:
+    """Bracket the tensor-core kernel of following calls with two CUDA
+    events (``torch.cuda.Event`` or raw handles); ``None, None`` stops."""
+    def h(e):
+        if e is None:
+            return None
+        return e if isinstance(e, int) else int(e.cuda_event)
+    library().gemm_profile_events(h(start_event), h(stop_event))
+
+
+def check(status: int) -> None:
+    if status != GEMM_OK:
+        raise GemmError(status)

@@ -1,0 +1,226 @@
+"""GPU parity: the CUDA library against the CPU oracle, element by element.
+
+int8 results must equal the oracle's exact sums bit for bit; bf16 results
+must satisfy |C - ref| <= 2^-8 |ref| + 2^-20 sum|a*b| for every element, and
+equal the nearest-even rounding of the exact sum bit for bit whenever the
+inputs make fp32 accumulation exact (integer-valued inputs).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2512_13282_gb300 import gemm as G
+from paper_2512_13282_gb300 import workloads as W
+from tests import gpu_util as U
+
+pytestmark = pytest.mark.gpu
+ROW, COL = G.GEMM_B_ROW_MAJOR_KxN, G.GEMM_B_COL_MAJOR_NxK
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2512_13282_gb300 import build
+    build.build()
+    G.library()
+
+
+def _inputs(dtype, M, N, K, layout, seed):
+    bshape = (K, N) if layout == ROW else (N, K)
+    if dtype == "int8":
+        return W.random_int8((M, K), seed), W.random_int8(bshape, seed + 1)
+    return W.random_bf16((M, K), seed), W.random_bf16(bshape, seed + 1)
+
+
+def _check(dtype, A, B, layout, C):
+    if dtype == "int8":
+        want = oracle.gemm_s8(A, B, layout)
+        assert np.abs(want).max(initial=0) < 2 ** 31
+        bad = np.argwhere(C.astype(np.int64) != want)
+        assert bad.size == 0, f"{len(bad)} mismatches, first at {bad[:5].tolist()}: " \
+                              f"{C[tuple(bad[0])]} vs {want[tuple(bad[0])]}"
+    else:
+        ref, mag = oracle.gemm_bf16(A, B, layout)
+        ok = oracle.bf16_within_bound(C, ref, mag)
+        bad = np.argwhere(~ok)
+        assert bad.size == 0, f"{len(bad)} out of bound, first at {bad[:5].tolist()}"
+        # diagnostic: most elements are the correctly rounded exact sum
+        exact = np.mean(C == oracle.rne_bf16(ref)) if C.size else 1.0
+        assert exact > 0.5, f"only {exact:.3f} of elements correctly rounded"
+
+
+SHAPES = [
+    (1, 1, 1), (5, 7, 3), (128, 256, 64), (129, 257, 65), (300, 520, 200),
+    (64, 1000, 1100), (257, 129, 2100), (130, 700, 4096), (1000, 1500, 3000),
+]
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("M,N,K", SHAPES, ids=[f"{m}x{n}x{k}" for m, n, k in SHAPES])
+def test_parity_shapes(dtype, layout, M, N, K):
+    A, B = _inputs(dtype, M, N, K, layout, seed=M * 7 + N * 3 + K)
+    C = U.run(dtype, A, B, layout)
+    _check(dtype, A, B, layout, C)
+
+
+SPLITK = [(16, 512, 4096), (128, 256, 8192), (1, 300, 5000), (3, 64, 20000)]
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("M,N,K", SPLITK, ids=[f"{m}x{n}x{k}" for m, n, k in SPLITK])
+def test_parity_split_k(dtype, layout, M, N, K):
+    A, B = _inputs(dtype, M, N, K, layout, seed=11)
+    C = U.run(dtype, A, B, layout)
+    _check(dtype, A, B, layout, C)
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("pads", [(1, 3, 5, 0, 0, 0), (0, 0, 0, 1, 1, 1), (8, 8, 8, 8, 8, 8),
+                                  (3, 0, 1, 0, 5, 3)],
+                         ids=["odd_ld", "odd_base", "wide_ld", "mixed"])
+def test_parity_leading_dims_and_offsets(dtype, layout, pads):
+    M, N, K = 200, 333, 777
+    pa, pb, pc, oa, ob, oc = pads
+    A, B = _inputs(dtype, M, N, K, layout, seed=21)
+    bcols = N if layout == ROW else K
+    C = U.run(dtype, A, B, layout, lda=K + pa, ldb=bcols + pb, ldc=N + pc, a_off=oa, b_off=ob, c_off=oc)
+    _check(dtype, A, B, layout, C)
+
+
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+def test_bf16_integer_inputs_bit_exact(layout):
+    """Integer-valued inputs in [-8, 8]: fp32 accumulation is exact in any
+    order, so C must be the correctly rounded exact sum, bit for bit."""
+    M, N, K = 300, 400, 1500
+    A = W.integer_bf16((M, K), 31)
+    B = W.integer_bf16((K, N) if layout == ROW else (N, K), 32)
+    C = U.run("bf16", A, B, layout)
+    ref, _ = oracle.gemm_bf16(A, B, layout)
+    assert np.array_equal(C, oracle.rne_bf16(ref))
+
+
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+def test_int8_all_minus128(layout):
+    """All -128: every 1024-long slab sums to exactly 2^24."""
+    M, N, K = 130, 260, 4096
+    A = np.full((M, K), -128, np.int8)
+    B = np.full((K, N) if layout == ROW else (N, K), -128, np.int8)
+    C = U.run("int8", A, B, layout)
+    assert (C == 16384 * K).all()
+
+
+def test_int8_edge_of_fp32_exactness():
+    """Slab sums of 1023 * 2^14 + 1 = 16760833: odd and just below 2^24, so
+    every bit of the fp32 significand is needed; signs vary by column."""
+    M, N, K = 128, 256, 3072
+    A = np.full((M, K), -128, np.int8)
+    A[:, 1023::1024] = 1
+    B = np.full((K, N), -128, np.int8)
+    B[1023::1024, :] = 1
+    sign = np.where(np.arange(N) % 3 == 0, -1, 1)
+    B = (B.astype(np.int16) * sign[None, :]).clip(-128, 127).astype(np.int8)
+    C = U.run("int8", A, B, ROW)
+    _check("int8", A, B, ROW, C)
+
+
+def test_int8_largest_exact_k():
+    """K = 131071 with all -128 gives 2147467264, the largest int32 the
+    exactness rule admits (split-K and slabs both involved)."""
+    M, N, K = 3, 5, 131071
+    A = np.full((M, K), -128, np.int8)
+    B = np.full((N, K), -128, np.int8)
+    C = U.run("int8", A, B, COL)
+    assert (C == 2147467264).all()
+    B2 = np.full((N, K), 127, np.int8)
+    C2 = U.run("int8", A, B2, COL)
+    assert (C2 == -16256 * K).all()
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+def test_k_zero_writes_zeros(dtype):
+    M, N = 70, 90
+    A = np.zeros((M, 0), np.int8 if dtype == "int8" else np.uint16)
+    B = np.zeros((0, N), A.dtype)
+    C = U.run(dtype, A, B, ROW)
+    assert (C == 0).all()
+
+
+def test_bf16_special_values():
+    M, N, K = 4, 300, 200
+    A = W.random_bf16((M, K), 41)
+    B = np.abs(W.random_bf16((K, N), 42).view(np.int16)).view(np.uint16)  # clear sign bits
+    A[0, 0] = 0x7FC0   # NaN
+    A[1, 5] = 0x7F80   # +inf
+    A[2, 7] = 0xFF80   # -inf
+    C = U.run("bf16", A, B, ROW)
+    _check("bf16", A, B, ROW, C)
+    c = oracle.bf16_bits_to_f64(C)
+    assert np.isnan(c[0]).all() and np.isposinf(c[1]).all() and np.isneginf(c[2]).all()
+
+
+def test_int8_k_too_large_rejected():
+    A = np.zeros((2, 131072), np.int8)
+    B = np.zeros((131072, 2), np.int8)
+    U.run("int8", A, B, ROW, expect=G.GEMM_ERR_UNSUPPORTED)
+
+
+def test_workspace_reuse_and_streams():
+    """Back-to-back calls of different sizes on a side stream reuse and grow
+    the workspace; results stay exact."""
+    s = torch.cuda.Stream()
+    for (M, N, K) in ((16, 512, 4096), (1, 3000, 9000), (300, 200, 100), (16, 512, 4096)):
+        A, B = _inputs("int8", M, N, K, COL, seed=M + N)
+        C = U.run("int8", A, B, COL, stream=s)
+        _check("int8", A, B, COL, C)
+
+
+def test_launch_counter_advances():
+    before = G.gemm_launch_count()
+    A, B = _inputs("bf16", 64, 64, 64, ROW, seed=5)
+    U.run("bf16", A, B, ROW)
+    assert G.gemm_launch_count() > before
+
+
+# ------------------------------------------------ full-size configurations
+
+def _sample_positions(M, N, BN=256, per_tile=3, cap=12000, seed=0):
+    """Tile corners and edges plus random interior points."""
+    rng = np.random.default_rng(seed)
+    rows = set()
+    for r0 in range(0, M, 128):
+        rows.update({r0, min(r0 + 127, M - 1)})
+    cols = set()
+    for c0 in range(0, N, 128):
+        cols.update({c0, min(c0 + 127, N - 1)})
+    rows, cols = np.array(sorted(rows)), np.array(sorted(cols))
+    rr, cc = np.meshgrid(rows, cols, indexing="ij")
+    r = np.concatenate([rr.ravel(), rng.integers(0, M, cap // 2), [M - 1]])
+    c = np.concatenate([cc.ravel(), rng.integers(0, N, cap // 2), [N - 1]])
+    if r.size > cap:
+        keep = rng.choice(r.size, cap, replace=False)
+        r, c = r[keep], c[keep]
+    return r.astype(np.int64), c.astype(np.int64)
+
+
+FULL = [g for w in W.WORKLOADS.values() for g in w.gemms]
+
+
+@pytest.mark.parametrize("g", FULL, ids=[g.name for g in FULL])
+def test_full_size_configs_sampled(g):
+    """Every GEMM of every workload at full size, in the launch configuration
+    the benchmark times: sampled outputs against the oracle, one by one."""
+    A, B = W.make_inputs(g)
+    C = U.run(g.dtype, A, B, g.layout)
+    r, c = _sample_positions(g.M, g.N, seed=g.M + g.N + g.K)
+    if g.dtype == "int8":
+        want = oracle.gemm_s8_entries(A, B, g.layout, r, c)
+        got = C[r, c].astype(np.int64)
+        assert np.array_equal(got, want), f"{np.sum(got != want)} of {r.size} sampled entries differ"
+    else:
+        ref, mag = oracle.gemm_bf16_entries(A, B, g.layout, r, c)
+        assert oracle.bf16_within_bound(C[r, c], ref, mag).all()
