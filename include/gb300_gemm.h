@@ -32,6 +32,7 @@
 #ifndef GB300_GEMM_H
 #define GB300_GEMM_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -83,6 +84,48 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K,
                                     const uint16_t *A, int64_t lda,
                                     const uint16_t *B, int64_t ldb, int b_layout,
                                     uint16_t *C, int64_t ldc, gemm_stream_t stream);
+
+/*
+ * Size of the fixed device scratch array used by gemm_s8s8_s32_noalloc.
+ * Every GPU on which the library's device code is loaded holds this much
+ * memory until the process exits.
+ */
+#define GEMM_NOALLOC_SCRATCH_BYTES ((size_t)128 << 20) /* 128 MiB */
+
+/*
+ * gemm_s8s8_s32_noalloc -- the same exact int8 GEMM as gemm_s8s8_s32, for
+ * callers that cannot let the library allocate device memory: an
+ * application whose own allocator holds nearly all device memory, a service
+ * enforcing a hard memory budget through its own allocator, or a
+ * latency-critical loop that cannot afford cudaMalloc/cudaFree and their
+ * synchronisation.  (The paper has no counterpart: it is an interface
+ * convenience of this library.)
+ *
+ *   Arguments, layouts, results and errors are those of gemm_s8s8_s32, and
+ *   the caller still owns A, B and C.  The operands' bf16 staging copies and
+ *   any split-K partial sums live in one static device array of
+ *   GEMM_NOALLOC_SCRATCH_BYTES bytes instead of the library's workspace; the
+ *   call never calls cudaMalloc, cudaFree or any other allocating routine.
+ *   Bytes needed: round256(2*M*K8) + round256(2*K8*N) for column-major B
+ *   (round256(2*M*K8) + round256(2*K*N8) for row-major B), plus
+ *   round256(4*S*M*N) when the planner splits K into S > 1 parts (S <= 16,
+ *   only for problems with fewer output tiles than SMs), where K8 and N8 are
+ *   K and N rounded up to multiples of 8.  A problem needing more returns
+ *   GEMM_ERR_UNSUPPORTED and launches nothing.
+ *
+ *   The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress) with that device current and caches it; make that
+ *   first call before any stream capture.  All calls share the one array and
+ *   it keeps whatever the last call left in it; every byte a call reads from
+ *   it is written earlier in the same call, so nothing needs clearing.  Calls
+ *   whose execution overlaps on the GPU (on different streams, or from
+ *   several host threads) race on the array and corrupt each other's
+ *   results: order them on one stream or synchronise between them.
+ */
+gemm_status_t gemm_s8s8_s32_noalloc(int64_t M, int64_t N, int64_t K,
+                                    const int8_t *A, int64_t lda,
+                                    const int8_t *B, int64_t ldb, int b_layout,
+                                    int32_t *C, int64_t ldc, gemm_stream_t stream);
 
 /* Human-readable name of a status code (static string, never NULL). */
 const char *gemm_status_string(gemm_status_t status);

@@ -355,3 +355,49 @@ void gemm_profile_events(void *start_event, void *stop_event) {
 }
 
 }  // extern "C"
+
+namespace gb300 {
+
+gemm_status_t validate_s8(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,
+                          int64_t ldb, int b_layout, const void *C, int64_t ldc) {
+  gemm_status_t s = check_common(M, N, K, A, lda, B, ldb, b_layout, C, ldc);
+  if (s != GEMM_OK) return s;
+  if (M > 0 && N > 0 && K > kMaxExactK) return GEMM_ERR_UNSUPPORTED;
+  return GEMM_OK;
+}
+
+// The int8 GEMM of gemm_s8s8_s32 with operand staging and split-K partials
+// placed in caller-provided device scratch [scratch, scratch + capacity)
+// instead of the library's workspace.  Returns GEMM_ERR_UNSUPPORTED, before
+// launching anything, when the problem needs more than `capacity` bytes.
+gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
+                                   const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
+                                   cudaStream_t st, void *scratch, size_t capacity) {
+  gemm_status_t s = validate_s8(M, N, K, A, lda, B, ldb, b_layout, C, ldc);
+  if (s != GEMM_OK || M == 0 || N == 0) return s;
+  DeviceState *d = nullptr;
+  if ((s = device_state(&d)) != GEMM_OK) return s;
+  if (K == 0) {
+    g_launches.fetch_add(1);
+    return launch_zero_fill(C, M, N, ldc, 4, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+  }
+  const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
+  Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
+  const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
+  const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;
+  const size_t a_off = 0;
+  const size_t b_off = align_up((size_t)M * lda_p * 2, 256);
+  const size_t part_off = align_up(b_off + (size_t)b_rows * ldb_p * 2, 256);
+  const size_t total = pl.p.splits > 1 ? align_up(part_off + (size_t)pl.p.splits * M * N * 4, 256) : part_off;
+  if (!scratch || total > capacity) return GEMM_ERR_UNSUPPORTED;
+  uint8_t *ws = static_cast<uint8_t *>(scratch);
+  uint16_t *Ab = reinterpret_cast<uint16_t *>(ws + a_off);
+  uint16_t *Bb = reinterpret_cast<uint16_t *>(ws + b_off);
+  g_launches.fetch_add(2);
+  if (launch_s8_to_bf16(A, M, K, lda, Ab, lda_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (launch_s8_to_bf16(B, b_rows, b_cols, ldb, Bb, ldb_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, pl.p.splits > 1 ? ws + part_off : nullptr, st);
+}
+
+}  // namespace gb300
+

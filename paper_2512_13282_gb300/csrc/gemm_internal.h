@@ -6,6 +6,7 @@
 
 #include <cstdint>
 
+#include "gb300_gemm.h"
 #include "gemm_tc.cuh"
 
 namespace gb300 {
@@ -43,5 +44,15 @@ cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, in
                                       uint16_t *C, int64_t ldc, int sms, cudaStream_t st);
 cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N,
                                      int32_t *C, int64_t ldc, int sms, cudaStream_t st);
+
+// Argument checks of the int8 entry points (no CUDA calls).
+gemm_status_t validate_s8(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,
+                          int64_t ldb, int b_layout, const void *C, int64_t ldc);
+
+// The int8 GEMM with its staging and split-K scratch in caller-provided
+// device memory of `capacity` bytes (gemm_api.cu; used by gemm_noalloc.cu).
+gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
+                                   const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
+                                   cudaStream_t st, void *scratch, size_t capacity);
 
 }  // namespace gb300

@@ -23,6 +23,8 @@ GEMM_ERR_UNSUPPORTED = 2
 GEMM_ERR_CUDA = 3
 GEMM_ERR_TIMEOUT = 4
 
+GEMM_NOALLOC_SCRATCH_BYTES = 128 << 20
+
 GEMM_B_ROW_MAJOR_KxN = 0
 GEMM_B_COL_MAJOR_NxK = 1
 
@@ -47,7 +49,7 @@ def library():
                                "paper_2512_13282_gb300.build.build() (no CPU fallback exists)")
         lib = ctypes.CDLL(LIB_PATH)
         i64, vp, ci = ctypes.c_int64, ctypes.c_void_p, ctypes.c_int
-        for name in ("gemm_s8s8_s32", "gemm_bf16_f32acc_bf16"):
+        for name in ("gemm_s8s8_s32", "gemm_bf16_f32acc_bf16", "gemm_s8s8_s32_noalloc"):
             f = getattr(lib, name)
             f.argtypes = [i64, i64, i64, vp, i64, vp, i64, ci, vp, i64, vp]
             f.restype = ci
@@ -86,6 +88,15 @@ def gemm_s8s8_s32(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int
     """C (int32, M x N) = A (int8, M x K) . B (int8, K x N), exact."""
     return int(library().gemm_s8s8_s32(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
                                        _ptr(C), ldc, _stream(stream)))
+
+
+def gemm_s8s8_s32_noalloc(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int:
+    """gemm_s8s8_s32 for callers that cannot let the library allocate device
+    memory: staging and split-K scratch live in a fixed 128 MiB device array
+    (GEMM_NOALLOC_SCRATCH_BYTES); larger problems return
+    GEMM_ERR_UNSUPPORTED.  Calls that overlap on the GPU race on that array."""
+    return int(library().gemm_s8s8_s32_noalloc(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
+                                               _ptr(C), ldc, _stream(stream)))
 
 
 def gemm_bf16_f32acc_bf16(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int:
