@@ -150,7 +150,7 @@ def run_ours(args, rank, world, dev):
     from paper_2512_13282_gb300 import gemm as G
     Bld.build()
     G.library()
-    wl = W.WORKLOADS[args.workload]
+    wl = select(args)
     cases = [GemmCase(g, dev) for g in wl.gemms]
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
@@ -284,14 +284,28 @@ def run_ours(args, rank, world, dev):
     return line
 
 
+def kernel_source_hash() -> str:
+    """Hash of the tensor-core kernel's sources: counters taken from an older
+    kernel are not reported as this kernel's."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("gemm_tc.cuh", "ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2512_13282_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
 def load_traffic(name):
-    """DRAM bytes per launch of the dominant kernel from the committed ncu
-    summary (profiles/traffic.json), or None when not captured for it."""
+    """DRAM bytes (read + write) per launch of the dominant kernel from the
+    committed ncu summary (profiles/traffic.json), or None when it was not
+    captured for this GEMM or the kernel source has changed since."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(p) as f:
             d = json.load(f)
-        return d.get(name)
+        if d.get("kernel_source_hash") != kernel_source_hash():
+            return None
+        return d.get("dram_bytes_per_launch", {}).get(name)
     except Exception:
         return None
 
@@ -307,6 +321,17 @@ def _oracle_rows(g: W.Gemm, A, B, rows):
         oracle.gemm_bf16(As, B, g.layout)
 
 
+def _calibrate_rows(g, A, B, budget):
+    """Rows of C the oracle computes in about `budget` seconds (the oracle
+    parallelises over rows, so calibrate on one row per thread)."""
+    import oracle
+    probe = min(g.M, max(1, oracle.num_threads()))
+    t0 = time.perf_counter()
+    _oracle_rows(g, A, B, probe)
+    t1 = time.perf_counter() - t0
+    return max(1, min(g.M, int(probe * budget / max(t1, 1e-6))))
+
+
 def cpu_baseline(wl, seconds):
     """Oracle throughput on whole rows of C of every GEMM of the workload,
     about `seconds` of CPU work in total."""
@@ -318,10 +343,7 @@ def cpu_baseline(wl, seconds):
     rows_used = []
     for g in wl.gemms:
         A, B = W.make_inputs(g)
-        t0 = time.perf_counter()
-        _oracle_rows(g, A, B, 1)
-        t1 = time.perf_counter() - t0
-        rows = max(1, min(g.M, int(budget / max(t1, 1e-6))))
+        rows = _calibrate_rows(g, A, B, budget)
         t0 = time.perf_counter()
         _oracle_rows(g, A, B, rows)
         dt = time.perf_counter() - t0
@@ -338,15 +360,10 @@ def run_reference(args, rank, world):
     samples (whole rows of C) of every GEMM of the workload."""
     import oracle
     oracle.build()
-    wl = W.WORKLOADS[args.workload]
+    wl = select(args)
     inputs = [W.make_inputs(g) for g in wl.gemms]
     per_step = args.cpu_seconds_per_step / len(wl.gemms)
-    rows = []
-    for g, (A, B) in zip(wl.gemms, inputs):
-        t0 = time.perf_counter()
-        _oracle_rows(g, A, B, 1)
-        t1 = time.perf_counter() - t0
-        rows.append(max(1, min(g.M, int(per_step / max(t1, 1e-6)))))
+    rows = [_calibrate_rows(g, A, B, per_step) for g, (A, B) in zip(wl.gemms, inputs)]
     for _ in range(args.warmup):
         for g, (A, B), r in zip(wl.gemms, inputs, rows):
             _oracle_rows(g, A, B, max(1, r // 8))
@@ -373,6 +390,17 @@ def run_reference(args, rank, world):
     }
 
 
+def select(args) -> W.Workload:
+    """The workload, optionally narrowed to the GEMMs named by --gemm."""
+    wl = W.WORKLOADS[args.workload]
+    if not args.gemm:
+        return wl
+    keep = tuple(g for g in wl.gemms if g.name in args.gemm)
+    if not keep:
+        raise SystemExit(f"--gemm matched nothing in {wl.name}: {[g.name for g in wl.gemms]}")
+    return W.Workload(wl.name, wl.description + " (subset: " + ", ".join(g.name for g in keep) + ")", keep)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -380,6 +408,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="square_sweep_512_4096", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--gemm", action="append", default=[],
+                    help="run only this GEMM of the workload (repeatable), e.g. bf16_4096x4096x4096_Bcol")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=16.0)
