@@ -289,7 +289,7 @@ def kernel_source_hash() -> str:
     kernel are not reported as this kernel's."""
     import hashlib
     h = hashlib.sha256()
-    for f in ("gemm_tc.cuh", "ptx.cuh"):
+    for f in ("gemm_tc.cuh", "gemm_tc2.cuh", "ptx.cuh"):
         with open(os.path.join(ROOT, "paper_2512_13282_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -412,7 +412,7 @@ def main():
                     help="run only this GEMM of the workload (repeatable), e.g. bf16_4096x4096x4096_Bcol")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=16.0)
+    ap.add_argument("--cpu-seconds", type=float, default=30.0)
     ap.add_argument("--cpu-seconds-per-step", type=float, default=6.0)
     args = ap.parse_args()
     if args.warmup < 3:

@@ -23,35 +23,50 @@ __device__ __forceinline__ uint32_t s8_to_bf16_bits(int v) {
   return __float_as_uint(static_cast<float>(v)) >> 16;
 }
 
-// Each thread converts 16 consecutive elements of a row.
-__global__ void s8_to_bf16_kernel(const int8_t *__restrict__ src, int64_t rows, int64_t cols,
-                                  int64_t ld_src, uint16_t *__restrict__ dst, int64_t ld_dst) {
-  const int64_t chunks_per_row = (cols + 15) / 16;
-  const int64_t total = rows * chunks_per_row;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = t / chunks_per_row;
-    const int64_t c = (t - r * chunks_per_row) * 16;
-    const int8_t *s = src + r * ld_src + c;
-    uint16_t *d = dst + r * ld_dst + c;
-    if (c + 16 <= cols && (reinterpret_cast<uintptr_t>(s) & 15) == 0 &&
-        (reinterpret_cast<uintptr_t>(d) & 15) == 0) {
-      const int4 raw = __ldg(reinterpret_cast<const int4 *>(s));
-      const uint32_t w[4] = {(uint32_t)raw.x, (uint32_t)raw.y, (uint32_t)raw.z, (uint32_t)raw.w};
-      uint32_t o[8];
+// Converts 16 int8 held in a uint4 to 16 bf16 bit patterns in two uint4.
+__device__ __forceinline__ void s8x16_to_bf16x16(const int4 raw, uint4 &lo, uint4 &hi) {
+  const uint32_t w[4] = {(uint32_t)raw.x, (uint32_t)raw.y, (uint32_t)raw.z, (uint32_t)raw.w};
+  uint32_t o[8];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int b0 = (int8_t)(w[i] & 0xFF), b1 = (int8_t)((w[i] >> 8) & 0xFF);
-        const int b2 = (int8_t)((w[i] >> 16) & 0xFF), b3 = (int8_t)(w[i] >> 24);
-        o[2 * i] = s8_to_bf16_bits(b0) | (s8_to_bf16_bits(b1) << 16);
-        o[2 * i + 1] = s8_to_bf16_bits(b2) | (s8_to_bf16_bits(b3) << 16);
-      }
-      uint4 *dv = reinterpret_cast<uint4 *>(d);
-      dv[0] = make_uint4(o[0], o[1], o[2], o[3]);
-      dv[1] = make_uint4(o[4], o[5], o[6], o[7]);
+  for (int i = 0; i < 4; ++i) {
+    const int b0 = (int8_t)(w[i] & 0xFF), b1 = (int8_t)((w[i] >> 8) & 0xFF);
+    const int b2 = (int8_t)((w[i] >> 16) & 0xFF), b3 = (int8_t)(w[i] >> 24);
+    o[2 * i] = s8_to_bf16_bits(b0) | (s8_to_bf16_bits(b1) << 16);
+    o[2 * i + 1] = s8_to_bf16_bits(b2) | (s8_to_bf16_bits(b3) << 16);
+  }
+  lo = make_uint4(o[0], o[1], o[2], o[3]);
+  hi = make_uint4(o[4], o[5], o[6], o[7]);
+}
+
+constexpr int kS8Chunk = 32;       // int8 elements per thread
+constexpr int kS8Threads = 128;    // threads per block: 4096 columns per block
+
+// blockIdx.z selects the job (A or B); blockIdx.y walks rows (strided by
+// gridDim.y); blockIdx.x covers 4096-column slices of a row; each thread
+// converts 32 consecutive elements.  Aligned full chunks use two 16-byte
+// loads and four 16-byte stores.
+__global__ void __launch_bounds__(kS8Threads) s8_to_bf16_pair_kernel(const S8Job a, const S8Job b) {
+  const S8Job j = blockIdx.z == 0 ? a : b;
+  const int64_t c = ((int64_t)blockIdx.x * kS8Threads + threadIdx.x) * kS8Chunk;
+  if (c >= j.cols) return;
+  const bool full = c + kS8Chunk <= j.cols;
+  for (int64_t r = blockIdx.y; r < j.rows; r += gridDim.y) {
+    const int8_t *src = j.src + r * j.ld_src + c;
+    uint16_t *dst = j.dst + r * j.ld_dst + c;
+    if (full && (reinterpret_cast<uintptr_t>(src) & 15) == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+      const int4 r0 = __ldg(reinterpret_cast<const int4 *>(src));
+      const int4 r1 = __ldg(reinterpret_cast<const int4 *>(src) + 1);
+      uint4 o0, o1, o2, o3;
+      s8x16_to_bf16x16(r0, o0, o1);
+      s8x16_to_bf16x16(r1, o2, o3);
+      uint4 *dv = reinterpret_cast<uint4 *>(dst);
+      dv[0] = o0;
+      dv[1] = o1;
+      dv[2] = o2;
+      dv[3] = o3;
     } else {
-      const int64_t n = cols - c < 16 ? cols - c : 16;
-      for (int64_t i = 0; i < n; ++i) d[i] = (uint16_t)s8_to_bf16_bits(s[i]);
+      const int64_t n = j.cols - c < kS8Chunk ? j.cols - c : kS8Chunk;
+      for (int64_t i = 0; i < n; ++i) dst[i] = (uint16_t)s8_to_bf16_bits(src[i]);
     }
   }
 }
@@ -105,10 +120,13 @@ __global__ void splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int spl
 
 }  // namespace
 
-cudaError_t launch_s8_to_bf16(const int8_t *src, int64_t rows, int64_t cols, int64_t ld_src,
-                              uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st) {
-  const int64_t work = rows * ((cols + 15) / 16);
-  s8_to_bf16_kernel<<<grid_for(work, 1, sms), kThreads, 0, st>>>(src, rows, cols, ld_src, dst, ld_dst);
+cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cudaStream_t st) {
+  (void)sms;
+  const int64_t per_block = (int64_t)kS8Threads * kS8Chunk;
+  const int64_t cols = a.cols > b.cols ? a.cols : b.cols;
+  const int64_t rows = a.rows > b.rows ? a.rows : b.rows;
+  const dim3 grid((unsigned)((cols + per_block - 1) / per_block), (unsigned)(rows < 65535 ? rows : 65535), 2);
+  s8_to_bf16_pair_kernel<<<grid, kS8Threads, 0, st>>>(a, b);
   return cudaGetLastError();
 }
 

@@ -7,6 +7,7 @@
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
@@ -144,23 +145,78 @@ struct Plan {
   int grid;
 };
 
-// Tile width, split-K factor and grid for an M x N x K problem on `sms` SMs.
-// BN = 256 when that still yields a full wave of tiles, else 128.  Split K
-// only when the tile count leaves most SMs idle, keeping >= 4 k-blocks per
-// split; the reduction then runs as a separate pass over fp32/int32 partials.
+// Kernel family, tile width, split-K factor and grid for an M x N x K
+// problem on `sms` SMs.
+//
+// Tile choice is the GB300 counterpart of the paper's balanced-tile search
+// (Sec. 4.5): the kernel runs in ceil(units / slots) rounds of one unit per
+// slot, where a slot is an SM (single-CTA kernel, 128 x BN tiles) or an SM
+// pair (pair kernel, 256 x BN tiles).  What one round costs was measured on
+// GB300 for long K (bf16, 4096^3..8192^3, relative to a 256 x 256 pair
+// round): it is nearly flat in BN, because the A tile, the pipeline latency
+// and the epilogue are paid by every tile whatever its width.  The family
+// and width with the least rounds * round cost win, the widest on a tie --
+// e.g. 4096^3 with B column-major: single-CTA 128 x 224 tiles in exactly 4
+// rounds of 152; 8192^3: pairs of 256 x 256 tiles.
+//
+// Split K only when the tile count leaves most slots idle and K is long; the
+// reduction then runs as a separate pass over fp32/int32 partials.
+int round_cost(bool pair, int bn) {
+  switch (bn) {
+    case 128: return pair ? 885 : 850;
+    case 192: return pair ? 950 : 920;
+    case 224: return pair ? 1000 : 980;
+    default: return pair ? 1000 : 1070;  // 256
+  }
+}
+
 Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms) {
   Plan pl{};
-  const int64_t tiles_m = ceil_div(M, kBM);
-  int bn = (N > 128 && tiles_m * ceil_div(N, 256) >= sms) ? 256 : 128;
+  const int pairs = pair_slots();
+  static const int kWidthsKMajor[] = {256, 224, 192, 128};
+  static const int kWidthsMNMajor[] = {256, 192, 128};
+  static const int kPairWidthsMNMajor[] = {256, 128};
   const int force_bn = env_int("GB300_GEMM_BN");
-  if (force_bn == 128 || force_bn == 256) bn = force_bn;
+  const char *force_pair_s = std::getenv("GB300_GEMM_PAIR");
+  const int force_pair = force_pair_s ? std::atoi(force_pair_s) : -1;
+  bool best_pair = false;
+  int best_bn = 128;
+  int64_t best_cost = -1;
+  for (int fam = 0; fam < 2; ++fam) {
+    const bool pair = fam == 1;
+    if (pair && (M <= kBM || pairs <= 0)) continue;  // the second CTA would only compute padding
+    if (force_pair >= 0 && (force_pair != 0) != pair) continue;
+    const int *widths = b_kmajor ? kWidthsKMajor : (pair ? kPairWidthsMNMajor : kWidthsMNMajor);
+    const int nw = b_kmajor ? 4 : (pair ? 2 : 3);
+    const int64_t slots = pair ? pairs : sms;
+    const int64_t tiles_m = ceil_div(M, pair ? 2 * kBM : kBM);
+    for (int i = 0; i < nw; ++i) {
+      const int bn = widths[i];
+      if (N <= 128 && bn != 128) continue;
+      if (force_bn > 0 && force_bn != bn) continue;
+      const int64_t rounds = ceil_div(tiles_m * ceil_div(N, bn), slots);
+      const int64_t cost = rounds * round_cost(pair, bn);
+      if (best_cost < 0 || cost < best_cost) {
+        best_cost = cost;
+        best_pair = pair;
+        best_bn = bn;
+      }
+    }
+  }
+  const bool pair = best_pair;
+  const int bn = best_bn;
+  const int64_t slots = pair ? pairs : sms;
+  const int64_t tiles_m = ceil_div(M, pair ? 2 * kBM : kBM);
   const int64_t tiles_n = ceil_div(N, bn);
   const int64_t tiles = tiles_m * tiles_n;
   const int64_t num_kb = ceil_div(K, kBK);
   int64_t splits = 1;
-  if (tiles * 2 <= sms && num_kb >= 8) {
-    splits = sms / tiles;
-    if (splits > num_kb / 4) splits = num_kb / 4;
+  // A split pays for an extra reduction launch (several microseconds), so
+  // only long reductions (K >= 2048) over few tiles are split, keeping >= 8
+  // k-blocks per split.
+  if (tiles * 2 <= slots && num_kb >= 32) {
+    splits = slots / tiles;
+    if (splits > num_kb / 8) splits = num_kb / 8;
     if (splits > 16) splits = 16;
     if (splits < 1) splits = 1;
   }
@@ -168,7 +224,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
   const int64_t kb_per = ceil_div(num_kb, splits);
   splits = ceil_div(num_kb, kb_per);
-  pl.v = TcVariant{bn, b_kmajor, epi};
+  pl.v = TcVariant{bn, b_kmajor, epi, pair};
   TcParams &p = pl.p;
   p.M = (int)M;
   p.N = (int)N;
@@ -181,7 +237,16 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   p.slab_kb = epi == kEpiS32 ? 1024 / kBK : (int)num_kb;
   p.group_m = 8;
   const int64_t units = tiles * splits;
-  pl.grid = (int)(units < sms ? units : sms);
+  const int64_t used = units < slots ? units : slots;
+  pl.grid = (int)(pair ? 2 * used : used);
+  static const bool debug = env_int("GB300_GEMM_DEBUG") != 0;
+  if (debug)
+    std::fprintf(stderr,
+                 "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d tiles=%lldx%lld splits=%lld grid=%d "
+                 "(SMs %d, co-resident pairs %d)\n",
+                 (long long)M, (long long)N, (long long)K, epi == kEpiS32 ? "int8" : "bf16",
+                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn, (long long)tiles_m, (long long)tiles_n,
+                 (long long)splits, pl.grid, sms, pairs);
   return pl;
 }
 
@@ -196,8 +261,11 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   TcParams &p = pl.p;
   CUtensorMap ta, tb;
   if (!encode_bf16_2d(&ta, A, (uint64_t)p.K, (uint64_t)p.M, (uint64_t)lda, kBK, kBM)) return GEMM_ERR_CUDA;
+  // K-major B boxes cover the CTA's share of the tile width: all of it, or
+  // half of it for a CTA pair.
+  const uint32_t b_rows = pl.v.pair ? pl.v.bn / 2 : pl.v.bn;
   const bool ok_b = pl.v.b_kmajor
-                        ? encode_bf16_2d(&tb, B, (uint64_t)p.K, (uint64_t)p.N, (uint64_t)ldb, kBK, pl.v.bn)
+                        ? encode_bf16_2d(&tb, B, (uint64_t)p.K, (uint64_t)p.N, (uint64_t)ldb, kBK, b_rows)
                         : encode_bf16_2d(&tb, B, (uint64_t)p.N, (uint64_t)p.K, (uint64_t)ldb, 64, kBK);
   if (!ok_b) return GEMM_ERR_CUDA;
   p.C = C;
@@ -208,8 +276,13 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   p.wait_limit_ns = wait_limit_ns();
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
-  cudaError_t e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, p, pl.grid, st)
-                                      : launch_tc_bf16(pl.v, ta, tb, p, pl.grid, st);
+  cudaError_t e;
+  if (pl.v.pair)
+    e = pl.v.epi == kEpiS32 ? launch_tc2_s32(pl.v, ta, tb, p, pl.grid, st)
+                            : launch_tc2_bf16(pl.v, ta, tb, p, pl.grid, st);
+  else
+    e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, p, pl.grid, st)
+                            : launch_tc_bf16(pl.v, ta, tb, p, pl.grid, st);
   g_launches.fetch_add(1);
   if (e != cudaSuccess) return GEMM_ERR_CUDA;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
@@ -306,9 +379,10 @@ gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K, const int8_t *A, in
   uint8_t *ws = static_cast<uint8_t *>(d->ws);
   uint16_t *Ab = reinterpret_cast<uint16_t *>(ws + L.a_off);
   uint16_t *Bb = reinterpret_cast<uint16_t *>(ws + L.b_off);
-  g_launches.fetch_add(2);
-  if (launch_s8_to_bf16(A, M, K, lda, Ab, lda_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
-  if (launch_s8_to_bf16(B, b_rows, b_cols, ldb, Bb, ldb_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  g_launches.fetch_add(1);
+  if (launch_s8_to_bf16_pair(S8Job{A, M, K, lda, Ab, lda_p}, S8Job{B, b_rows, b_cols, ldb, Bb, ldb_p}, d->sms,
+                             st) != cudaSuccess)
+    return GEMM_ERR_CUDA;
   return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, pl.p.splits > 1 ? ws + L.part_off : nullptr, st);
 }
 
@@ -393,9 +467,10 @@ gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t
   uint8_t *ws = static_cast<uint8_t *>(scratch);
   uint16_t *Ab = reinterpret_cast<uint16_t *>(ws + a_off);
   uint16_t *Bb = reinterpret_cast<uint16_t *>(ws + b_off);
-  g_launches.fetch_add(2);
-  if (launch_s8_to_bf16(A, M, K, lda, Ab, lda_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
-  if (launch_s8_to_bf16(B, b_rows, b_cols, ldb, Bb, ldb_p, d->sms, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  g_launches.fetch_add(1);
+  if (launch_s8_to_bf16_pair(S8Job{A, M, K, lda, Ab, lda_p}, S8Job{B, b_rows, b_cols, ldb, Bb, ldb_p}, d->sms,
+                             st) != cudaSuccess)
+    return GEMM_ERR_CUDA;
   return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, pl.p.splits > 1 ? ws + part_off : nullptr, st);
 }
 

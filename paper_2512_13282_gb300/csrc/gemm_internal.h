@@ -13,25 +13,35 @@ namespace gb300 {
 
 // One compiled variant of the tcgen05 kernel.
 struct TcVariant {
-  int bn;        // 128 or 256
+  int bn;        // tile width (see the instantiation files for the compiled set)
   bool b_kmajor; // B stored N x K (K contiguous)
   int epi;       // kEpiBf16 or kEpiS32
+  bool pair;     // CTA-pair kernel (256-row tiles, cta_group::2) or single CTA (128 rows)
 };
-
-// Shared-memory bytes and threads of a variant (for occupancy/launch).
-int tc_smem_bytes(const TcVariant &v);
-int tc_threads(const TcVariant &v);
 
 // Launch the persistent tcgen05 GEMM kernel (gemm_tc_bf16.cu / gemm_tc_s32.cu).
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const TcParams &p, int grid, cudaStream_t st);
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                           const TcParams &p, int grid, cudaStream_t st);
+// Number of CTA pairs that can be resident at once (0 if unknown).
+int pair_slots();
+// The CTA-pair kernel (gemm_tc2_bf16.cu / gemm_tc2_s32.cu); grid is even.
+cudaError_t launch_tc2_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
+                            const TcParams &p, int grid, cudaStream_t st);
+cudaError_t launch_tc2_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
+                           const TcParams &p, int grid, cudaStream_t st);
 
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
-// int8 -> bf16 (exact), rows x cols, arbitrary source leading dimension.
-cudaError_t launch_s8_to_bf16(const int8_t *src, int64_t rows, int64_t cols, int64_t ld_src,
-                              uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st);
+// int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is
+// rows x cols with an arbitrary source leading dimension.
+struct S8Job {
+  const int8_t *src;
+  int64_t rows, cols, ld_src;
+  uint16_t *dst;
+  int64_t ld_dst;
+};
+cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cudaStream_t st);
 // bf16 copy into an aligned buffer (re-pitching a misaligned operand).
 cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int64_t ld_src,
                             uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st);

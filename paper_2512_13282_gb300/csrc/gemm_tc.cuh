@@ -62,19 +62,30 @@ struct TcParams {
   uint64_t wait_limit_ns;
 };
 
+__host__ __device__ constexpr uint32_t pow2_at_least(uint32_t x) {
+  uint32_t p = 32;
+  while (p < x) p <<= 1;
+  return p;
+}
+
 template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
 struct TcCfg {
-  static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256, a multiple of 64");
+  // MMA N for M = 128 is a multiple of 16 up to 256; the epilogue moves 32
+  // columns per TMEM load; an MN-major B tile is assembled from 64-wide boxes.
+  static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256, a multiple of 32");
+  static_assert(B_KMAJOR || BN % 64 == 0, "MN-major B needs BN a multiple of 64");
   static_assert(EPI_WARPS == 4 || EPI_WARPS == 8, "epilogue is one or two warpgroups");
   static constexpr uint32_t kBBytes = BN * kRowBytes;
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
-  static constexpr uint32_t kTmemCols = 2 * BN;  // two fp32 accumulators
+  static constexpr uint32_t kTmemCols = pow2_at_least(2 * BN);  // two fp32 accumulators
   static constexpr int kThreads = (2 + EPI_WARPS) * 32;
   static constexpr int kColsPerThread = BN / (EPI_WARPS / 4);
+  static_assert(kColsPerThread % 16 == 0, "epilogue chunks are 32 columns, plus one of 16");
   static constexpr uint32_t kBarOffset = STAGES * kStageBytes;
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
-  static_assert(kTmemCols == 256 || kTmemCols == 512 || kTmemCols == 128, "TMEM columns");
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
+  static_assert(kTmemCols <= 512, "TMEM has 512 columns");
 };
 
 struct Unit {
@@ -106,18 +117,44 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&v);
 }
 
-// Store 32 consecutive 32-bit words of one row (fp32 partials or int32).
-__device__ __forceinline__ void store_row32(uint32_t *dst, int col, int N, bool vec,
-                                            const uint32_t (&v)[32]) {
-  if (vec && col + 32 <= N) {
+// Store W (16 or 32) consecutive 32-bit words of one row (fp32 partials or
+// int32), vectorised when the row is 16-byte aligned and fully inside N.
+template <int W>
+__device__ __forceinline__ void store_words(uint32_t *dst, int col, int N, bool vec, const uint32_t (&v)[W]) {
+  if (vec && col + W <= N) {
     uint4 *d = reinterpret_cast<uint4 *>(dst + col);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) d[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    for (int i = 0; i < W / 4; ++i) d[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
   } else {
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
+    for (int i = 0; i < W; ++i)
       if (col + i < N) dst[col + i] = v[i];
   }
+}
+
+// Round W fp32 accumulator words to bf16 (nearest even) and store them.
+template <int W>
+__device__ __forceinline__ void store_bf16(uint16_t *dst, int col, int N, bool vec, const uint32_t (&r)[W]) {
+  uint32_t h[W / 2];
+#pragma unroll
+  for (int i = 0; i < W / 2; ++i) h[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+  if (vec && col + W <= N) {
+    uint4 *d = reinterpret_cast<uint4 *>(dst + col);
+#pragma unroll
+    for (int i = 0; i < W / 8; ++i) d[i] = make_uint4(h[4 * i], h[4 * i + 1], h[4 * i + 2], h[4 * i + 3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < W; ++i)
+      if (col + i < N) dst[col + i] = static_cast<uint16_t>(h[i >> 1] >> (16 * (i & 1)));
+  }
+}
+
+template <int W>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
+  if constexpr (W == 32)
+    tmem_ld_32x32b_x32(taddr, r);
+  else
+    tmem_ld_32x32b_x16(taddr, r);
 }
 
 template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
@@ -281,10 +318,18 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t r[32];
-            tmem_ld_32x32b_x32(t0 + c * 32, r);
+            tmem_ld<32>(t0 + c * 32, r);
             tmem_ld_wait();
 #pragma unroll
             for (int i = 0; i < 32; ++i) acc[c * 32 + i] += __float2int_rn(__uint_as_float(r[i]));
+          }
+          if constexpr (CPT % 32 != 0) {
+            constexpr int kTail = (CPT / 32) * 32;
+            uint32_t r[16];
+            tmem_ld<16>(t0 + kTail, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) acc[kTail + i] += __float2int_rn(__uint_as_float(r[i]));
           }
           tc_fence_before_sync();
           mbar_arrive(acce_bar(b));
@@ -300,7 +345,14 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
             uint32_t v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
-            store_row32(dst, col0 + c * 32, p.N, vec, v);
+            store_words<32>(dst, col0 + c * 32, p.N, vec, v);
+          }
+          if constexpr (CPT % 32 != 0) {
+            constexpr int kTail = (CPT / 32) * 32;
+            uint32_t v[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
+            store_words<16>(dst, col0 + kTail, p.N, vec, v);
           }
         }
       } else {
@@ -311,30 +363,30 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
         }
         tc_fence_after_sync();
         const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
+uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                               : nullptr;
 #pragma unroll 1
         for (int c = 0; c < CPT / 32; ++c) {
           uint32_t r[32];
-          tmem_ld_32x32b_x32(t0 + c * 32, r);
+          tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
           if (!row_ok) continue;
-          const int col = col0 + c * 32;
-          if (split) {
-            uint32_t *dst = reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N;
-            store_row32(dst, col, p.N, ws_vec, r);
-          } else {
-            uint16_t *dst = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
-            uint32_t h[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) h[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
-            if (p.c_vec && col + 32 <= p.N) {
-              uint4 *d = reinterpret_cast<uint4 *>(dst + col);
-#pragma unroll
-              for (int i = 0; i < 4; ++i) d[i] = make_uint4(h[4 * i], h[4 * i + 1], h[4 * i + 2], h[4 * i + 3]);
-            } else {
-#pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (col + i < p.N) dst[col + i] = static_cast<uint16_t>(h[i >> 1] >> (16 * (i & 1)));
-            }
+          if (split)
+            store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, r);
+          else
+            store_bf16<32>(crow, col0 + c * 32, p.N, p.c_vec != 0, r);
+        }
+        if constexpr (CPT % 32 != 0) {
+          constexpr int kTail = (CPT / 32) * 32;
+          uint32_t r[16];
+          tmem_ld<16>(t0 + kTail, r);
+          tmem_ld_wait();
+          if (row_ok) {
+            if (split)
+              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, r);
+            else
+              store_bf16<16>(crow, col0 + kTail, p.N, p.c_vec != 0, r);
           }
         }
         tc_fence_before_sync();

@@ -1,0 +1,54 @@
+// Instantiations of the CTA-pair tcgen05 kernel with the bf16 epilogue.
+#include "gemm_tc2_launch.cuh"
+
+namespace gb300 {
+
+// Pair tile widths (256 x BN per pair; BN/2 columns of B per CTA): 256 and
+// 128 for either B layout, 224 and 192 for B column-major.
+cudaError_t launch_tc2_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
+                            const TcParams &p, int grid, cudaStream_t st) {
+  if (v.b_kmajor) {
+    switch (v.bn) {
+      case 256: return launch_pair<256, 6, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 224: return launch_pair<224, 7, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 192: return launch_pair<192, 7, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 128: return launch_pair<128, 8, true, kEpiBf16, 4>(a, b, p, grid, st);
+    }
+  } else {
+    switch (v.bn) {
+      case 256: return launch_pair<256, 6, false, kEpiBf16, 4>(a, b, p, grid, st);
+      case 128: return launch_pair<128, 8, false, kEpiBf16, 4>(a, b, p, grid, st);
+    }
+  }
+  return cudaErrorInvalidValue;
+}
+
+int pair_slots() {
+  // Co-resident SM pairs for a kernel holding one CTA per SM (all pair
+  // variants use > 113 KB of shared memory), queried once per device.
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] > 0) return cached[dev];
+  using Cfg = Tc2Cfg<256, 6, true, kEpiBf16, 4>;
+  auto kern = gemm_tc2_kernel<256, 6, true, kEpiBf16, 4>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2, 1, 1);
+  cfg.blockDim = dim3(Cfg::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) return 0;
+  cached[dev] = n;
+  return n;
+}
+
+}  // namespace gb300

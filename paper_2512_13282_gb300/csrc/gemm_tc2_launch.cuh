@@ -1,0 +1,38 @@
+// gemm_tc2_launch.cuh -- cluster launch of the CTA-pair kernel (included by
+// the instantiation translation units).
+#pragma once
+#include "gemm_internal.h"
+#include "gemm_tc2.cuh"
+
+namespace gb300 {
+
+template <int BN, int STAGES, bool KM, int EPI, int EW>
+cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const TcParams &p, int grid,
+                        cudaStream_t st) {
+  using Cfg = Tc2Cfg<BN, STAGES, KM, EPI, EW>;
+  auto kern = gemm_tc2_kernel<BN, STAGES, KM, EPI, EW>;
+  static bool opted_in[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || !opted_in[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) opted_in[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);  // even: a whole number of pairs
+  cfg.blockDim = dim3(Cfg::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a, b, p);
+}
+
+}  // namespace gb300

@@ -9,20 +9,40 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParam
                        cudaStream_t st) {
   using Cfg = TcCfg<BN, STAGES, KM, EPI, EW>;
   auto kern = gemm_tc_kernel<BN, STAGES, KM, EPI, EW>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+  // the shared-memory opt-in is per device and kernel: set it once
+  static bool opted_in[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || !opted_in[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) opted_in[dev] = true;
+  }
   kern<<<grid, Cfg::kThreads, Cfg::kSmemBytes, st>>>(a, b, p);
   return cudaGetLastError();
 }
 }  // namespace
 
+// Tile widths compiled for the bf16 epilogue: 128 (6 stages), 192 (5),
+// 224 (5, B column-major only), 256 (4).
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const TcParams &p, int grid, cudaStream_t st) {
-  if (v.bn == 256)
-    return v.b_kmajor ? launch_one<256, 4, true, kEpiBf16, 4>(a, b, p, grid, st)
-                      : launch_one<256, 4, false, kEpiBf16, 4>(a, b, p, grid, st);
-  return v.b_kmajor ? launch_one<128, 6, true, kEpiBf16, 4>(a, b, p, grid, st)
-                    : launch_one<128, 6, false, kEpiBf16, 4>(a, b, p, grid, st);
+  if (v.b_kmajor) {
+    switch (v.bn) {
+      case 256: return launch_one<256, 4, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 224: return launch_one<224, 5, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 192: return launch_one<192, 5, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 128: return launch_one<128, 6, true, kEpiBf16, 4>(a, b, p, grid, st);
+    }
+  } else {
+    switch (v.bn) {
+      case 256: return launch_one<256, 4, false, kEpiBf16, 4>(a, b, p, grid, st);
+      case 192: return launch_one<192, 5, false, kEpiBf16, 4>(a, b, p, grid, st);
+      case 128: return launch_one<128, 6, false, kEpiBf16, 4>(a, b, p, grid, st);
+    }
+  }
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace gb300

@@ -9,30 +9,37 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParam
                        cudaStream_t st) {
   using Cfg = TcCfg<BN, STAGES, KM, EPI, EW>;
   auto kern = gemm_tc_kernel<BN, STAGES, KM, EPI, EW>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+  // the shared-memory opt-in is per device and kernel: set it once
+  static bool opted_in[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || !opted_in[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) opted_in[dev] = true;
+  }
   kern<<<grid, Cfg::kThreads, Cfg::kSmemBytes, st>>>(a, b, p);
   return cudaGetLastError();
 }
 }  // namespace
 
+// Tile widths compiled for the int32 epilogue: 128 (one epilogue warpgroup,
+// 128 int32 accumulators per thread), 192, 224 (B column-major only) and 256
+// (two warpgroups, 96 / 112 / 128 per thread).
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                           const TcParams &p, int grid, cudaStream_t st) {
-  if (v.bn == 256)
-    return v.b_kmajor ? launch_one<256, 4, true, kEpiS32, 8>(a, b, p, grid, st)
-                      : launch_one<256, 4, false, kEpiS32, 8>(a, b, p, grid, st);
-  return v.b_kmajor ? launch_one<128, 6, true, kEpiS32, 4>(a, b, p, grid, st)
-                    : launch_one<128, 6, false, kEpiS32, 4>(a, b, p, grid, st);
-}
-
-int tc_smem_bytes(const TcVariant &v) {
-  if (v.bn == 256) return (int)TcCfg<256, 4, true, kEpiS32, 8>::kSmemBytes;
-  return (int)TcCfg<128, 6, true, kEpiS32, 4>::kSmemBytes;
-}
-
-int tc_threads(const TcVariant &v) {
-  if (v.epi == kEpiS32 && v.bn == 256) return TcCfg<256, 4, true, kEpiS32, 8>::kThreads;
-  return TcCfg<128, 6, true, kEpiBf16, 4>::kThreads;
+  switch (v.bn) {
+    case 256: return v.b_kmajor ? launch_one<256, 4, true, kEpiS32, 8>(a, b, p, grid, st)
+                                : launch_one<256, 4, false, kEpiS32, 8>(a, b, p, grid, st);
+    case 224: return v.b_kmajor ? launch_one<224, 5, true, kEpiS32, 8>(a, b, p, grid, st)
+                                : cudaErrorInvalidValue;
+    case 192: return v.b_kmajor ? launch_one<192, 5, true, kEpiS32, 8>(a, b, p, grid, st)
+                                : launch_one<192, 5, false, kEpiS32, 8>(a, b, p, grid, st);
+    case 128: return v.b_kmajor ? launch_one<128, 6, true, kEpiS32, 4>(a, b, p, grid, st)
+                                : launch_one<128, 6, false, kEpiS32, 4>(a, b, p, grid, st);
+  }
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace gb300

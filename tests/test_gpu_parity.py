@@ -224,3 +224,20 @@ def test_full_size_configs_sampled(g):
     else:
         ref, mag = oracle.gemm_bf16_entries(A, B, g.layout, r, c)
         assert oracle.bf16_within_bound(C[r, c], ref, mag).all()
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("bn", [128, 192, 224, 256])
+@pytest.mark.parametrize("pair", ["0", "1"], ids=["single", "pair"])
+def test_parity_every_tile_width(dtype, layout, bn, pair, monkeypatch):
+    """Each compiled kernel family (one CTA per 128-row tile, or CTA pairs
+    per 256-row tile) and tile width -- the planner normally picks one per
+    shape -- on ragged multi-tile shapes, with and without split-K."""
+    monkeypatch.setenv("GB300_GEMM_BN", str(bn))
+    monkeypatch.setenv("GB300_GEMM_PAIR", pair)
+    for (M, N, K, splits) in ((300, 700, 1500, "1"), (130, 450, 3000, "3")):
+        monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
+        A, B = _inputs(dtype, M, N, K, layout, seed=bn + M)
+        C = U.run(dtype, A, B, layout)
+        _check(dtype, A, B, layout, C)
