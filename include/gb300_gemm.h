@@ -146,6 +146,17 @@ void gemm_release_resources(void);
 uint64_t gemm_launch_count(void);
 
 /*
+ * Failure-detection self-test (a diagnostic; the paper has no counterpart).
+ * Launches one thread that waits, with the same bounded mbarrier wait the
+ * GEMM kernels use, on a barrier nothing arrives on.  After `limit_ns`
+ * (1 .. 1e9 ns, else GEMM_ERR_INVALID_ARG) the wait gives up and records
+ * GEMM_ERR_TIMEOUT in the device error word; gemm_device_status() then
+ * reports (and clears) it.  The kernel ends normally and the context stays
+ * usable.  Returns GEMM_OK once the probe is launched.
+ */
+gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream);
+
+/*
  * Profiling aid.  With both arguments non-NULL (cudaEvent_t handles created
  * by the caller), every following GEMM call records `start_event` on its
  * stream just before launching its tensor-core kernel and `stop_event` just

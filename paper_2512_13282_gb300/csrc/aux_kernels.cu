@@ -118,7 +118,27 @@ __global__ void splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int spl
   }
 }
 
+// One thread waits, with the GEMM kernels' bounded wait, on an mbarrier that
+// nothing will ever arrive on: the wait gives up after limit_ns and records
+// the timeout in the device error word, exactly as a stalled GEMM would.
+__global__ void wait_timeout_probe_kernel(uint32_t *err, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_addr(&bar), 1);
+    abort_flag = 0u;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) (void)mbar_wait(smem_addr(&bar), 0, &abort_flag, err, limit_ns);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStream_t st) {
+  wait_timeout_probe_kernel<<<1, 32, 0, st>>>(err, limit_ns);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cudaStream_t st) {
   (void)sms;

@@ -32,6 +32,8 @@ struct DeviceState {
   uint32_t *err = nullptr;
   void *ws = nullptr;
   size_t ws_bytes = 0;
+  uint32_t *tickets = nullptr;  // zeroed counters of the small-M kernel
+  size_t tickets_count = 0;
 };
 
 std::mutex g_mu;
@@ -103,6 +105,24 @@ gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
 int env_int(const char *name) {
   const char *s = std::getenv(name);
   return s ? std::atoi(s) : 0;
+}
+
+// Grow the zeroed ticket counters of the small-M kernel to `count`.
+gemm_status_t ensure_tickets(DeviceState &d, size_t count, cudaStream_t st) {
+  if (count <= d.tickets_count) return GEMM_OK;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (count <= d.tickets_count) return GEMM_OK;
+  if (d.tickets && cudaFreeAsync(d.tickets, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  d.tickets = nullptr;
+  d.tickets_count = 0;
+  const size_t n = count < 1024 ? 1024 : count;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&d.tickets), n * sizeof(uint32_t), st) != cudaSuccess ||
+      cudaMemsetAsync(d.tickets, 0, n * sizeof(uint32_t), st) != cudaSuccess) {
+    d.tickets = nullptr;
+    return GEMM_ERR_CUDA;
+  }
+  d.tickets_count = n;
+  return GEMM_OK;
 }
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -298,6 +318,54 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   return GEMM_OK;
 }
 
+// Largest M sent to the CUDA-core small-M kernel: there every B element is
+// used at most a few times and streaming B once is the cost.  Measured on
+// GB300 against the tensor-core path (N = 4096..11008, K = 4096): int8
+// through dp4a, which also skips the staging pass, wins up to M = 8; bf16,
+// accumulating with fp32 FMAs, only up to M = 2.
+// GB300_GEMM_SKINNY_MAX_M overrides (0 disables the kernel).
+int skinny_max_m(bool int8) {
+  const char *s = std::getenv("GB300_GEMM_SKINNY_MAX_M");
+  if (s) {
+    const int v = std::atoi(s);
+    return v < 0 ? 0 : (v > 16 ? 16 : v);
+  }
+  return int8 ? 8 : 2;
+}
+
+gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const void *A, int64_t lda,
+                         const void *B, int64_t ldb, bool b_kmajor, void *C, int64_t ldc, bool int8,
+                         cudaStream_t st) {
+  const bool row_b = !b_kmajor;
+  const int64_t strips = ceil_div(N, row_b ? 256 : 32);
+  SkinnyParams p{};
+  skinny_split(K, strips, d.sms, (int)M, int8 ? 1 : 2, &p.kb, &p.ks);
+  p.A = A;
+  p.lda = lda;
+  p.B = B;
+  p.ldb = ldb;
+  p.C = C;
+  p.ldc = ldc;
+  p.M = (int)M;
+  p.N = N;
+  p.K = K;
+  const int esize = int8 ? 1 : 2;
+  const uintptr_t bb = reinterpret_cast<uintptr_t>(B);
+  if (row_b && int8)
+    p.b_vec = (bb % 8 == 0) && (ldb % 8 == 0);
+  else
+    p.b_vec = (bb % 16 == 0) && ((ldb * esize) % 16 == 0);
+  gemm_status_t s;
+  if (p.ks > 1) {
+    if ((s = ensure_workspace(d, (size_t)p.ks * M * N * 4, st)) != GEMM_OK) return s;
+    if ((s = ensure_tickets(d, (size_t)strips, st)) != GEMM_OK) return s;
+    p.ws = d.ws;
+    p.tickets = d.tickets;
+  }
+  g_launches.fetch_add(1);
+  return launch_skinny(p, int8, row_b, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+}
+
 }  // namespace
 
 extern "C" {
@@ -315,6 +383,8 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
     return launch_zero_fill(C, M, N, ldc, 2, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
   }
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
+  if (M <= skinny_max_m(false))
+    return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, false, st);
   Plan pl = make_plan(M, N, K, b_kmajor, kEpiBf16, d->sms);
   // TMA needs 16-byte aligned bases and row pitches; re-pitch an operand
   // that is not, into the workspace.
@@ -363,6 +433,8 @@ gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K, const int8_t *A, in
     return launch_zero_fill(C, M, N, ldc, 4, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
   }
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
+  if (M <= skinny_max_m(true))
+    return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, true, st);
   Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
   // Stage both operands as bf16 (exact for int8) with 16-byte aligned rows.
   const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
@@ -419,9 +491,23 @@ void gemm_release_resources(void) {
   if (d.ws) cudaFree(d.ws);
   d.ws = nullptr;
   d.ws_bytes = 0;
+  if (d.tickets) cudaFree(d.tickets);
+  d.tickets = nullptr;
+  d.tickets_count = 0;
 }
 
 uint64_t gemm_launch_count(void) { return g_launches.load(); }
+
+gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream) {
+  if (limit_ns == 0 || limit_ns > 1000000000ull) return GEMM_ERR_INVALID_ARG;
+  DeviceState *d = nullptr;
+  gemm_status_t s = device_state(&d);
+  if (s != GEMM_OK) return s;
+  g_launches.fetch_add(1);
+  return launch_wait_timeout_probe(d->err, limit_ns, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? GEMM_OK
+             : GEMM_ERR_CUDA;
+}
 
 void gemm_profile_events(void *start_event, void *stop_event) {
   g_prof_start = static_cast<cudaEvent_t>(start_event);

@@ -45,6 +45,9 @@ cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cuda
 // bf16 copy into an aligned buffer (re-pitching a misaligned operand).
 cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int64_t ld_src,
                             uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st);
+// One-thread kernel whose bounded mbarrier wait is made to expire
+// (failure-detection self-test).
+cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStream_t st);
 // Fill an M x N block of 16- or 32-bit elements with zero.
 cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esize, int sms,
                              cudaStream_t st);
@@ -64,5 +67,24 @@ gemm_status_t validate_s8(int64_t M, int64_t N, int64_t K, const void *A, int64_
 gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
                                    const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
                                    cudaStream_t st, void *scratch, size_t capacity);
+
+// Small-M GEMM on the CUDA cores (gemm_skinny.cu).  M <= 16.
+struct SkinnyParams {
+  const void *A;
+  int64_t lda;
+  const void *B;
+  int64_t ldb;
+  void *C;
+  int64_t ldc;
+  int M;
+  int64_t N, K;
+  int kb;              // rows of K per block slice (multiple of 32)
+  int ks;              // slices (blocks per column strip)
+  int b_vec;           // B rows allow 16-byte (8-byte for row-major int8) loads
+  void *ws;            // ks x M x N 32-bit partials (ks > 1)
+  uint32_t *tickets;   // one zeroed counter per column strip (ks > 1)
+};
+void skinny_split(int64_t K, int64_t strips, int sms, int m_rows, int esize, int *kb, int *ks);
+cudaError_t launch_skinny(const SkinnyParams &p, bool int8, bool row_b, cudaStream_t st);
 
 }  // namespace gb300

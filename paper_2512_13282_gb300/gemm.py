@@ -61,6 +61,8 @@ def library():
         lib.gemm_release_resources.restype = None
         lib.gemm_launch_count.argtypes = []
         lib.gemm_launch_count.restype = ctypes.c_uint64
+        lib.gemm_selftest_wait_timeout.argtypes = [ctypes.c_uint64, vp]
+        lib.gemm_selftest_wait_timeout.restype = ci
         lib.gemm_profile_events.argtypes = [vp, vp]
         lib.gemm_profile_events.restype = None
         _lib = lib
@@ -119,6 +121,11 @@ def gemm_release_resources() -> None:
 
 def gemm_launch_count() -> int:
     return int(library().gemm_launch_count())
+
+
+def gemm_selftest_wait_timeout(limit_ns: int, stream=None) -> int:
+    """Launch the bounded-wait probe that is made to time out; see the header."""
+    return int(library().gemm_selftest_wait_timeout(int(limit_ns), _stream(stream)))
 
 
 def gemm_profile_events(start_event, stop_event) -> None:

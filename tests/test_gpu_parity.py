@@ -241,3 +241,47 @@ def test_parity_every_tile_width(dtype, layout, bn, pair, monkeypatch):
         A, B = _inputs(dtype, M, N, K, layout, seed=bn + M)
         C = U.run(dtype, A, B, layout)
         _check(dtype, A, B, layout, C)
+
+
+SKINNY = [(1, 1, 1), (1, 11008, 4096), (2, 257, 777), (3, 1000, 4100), (5, 300, 64), (8, 4096, 4096),
+          (13, 555, 2049), (16, 4096, 4096), (16, 96, 20000)]
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("M,N,K", SKINNY, ids=[f"{m}x{n}x{k}" for m, n, k in SKINNY])
+@pytest.mark.parametrize("path", ["auto", "cudacore", "tensor"])
+def test_parity_small_m(dtype, layout, M, N, K, path, monkeypatch):
+    """M <= 16: the CUDA-core small-M kernel (forced, or as the planner
+    routes it) and the tensor-core path (forced), full comparison."""
+    if path == "cudacore":
+        monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "16")
+    elif path == "tensor":
+        monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    A, B = _inputs(dtype, M, N, K, layout, seed=M * 31 + N)
+    C = U.run(dtype, A, B, layout)
+    _check(dtype, A, B, layout, C)
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+def test_small_m_misaligned_and_repeated(dtype, layout, monkeypatch):
+    """Odd leading dimensions and bases take the scalar load paths; calls in
+    a row reuse the self-resetting reduction counters."""
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "16")
+    for rep, (M, N, K) in enumerate(((7, 333, 3001), (16, 1024, 8192), (7, 333, 3001))):
+        A, B = _inputs(dtype, M, N, K, layout, seed=rep)
+        bcols = N if layout == ROW else K
+        C = U.run(dtype, A, B, layout, lda=K + 3, ldb=bcols + 1, ldc=N + 2, a_off=1, b_off=3, c_off=1)
+        _check(dtype, A, B, layout, C)
+
+
+def test_small_m_int8_extremes(monkeypatch):
+    """dp4a exactness at the int32 edge: K = 131071 of (-128)(-128)."""
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "16")
+    for layout in (ROW, COL):
+        M, N, K = 2, 40, 131071
+        A = np.full((M, K), -128, np.int8)
+        B = np.full((K, N) if layout == ROW else (N, K), -128, np.int8)
+        C = U.run("int8", A, B, layout)
+        assert (C == 2147467264).all()
