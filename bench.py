@@ -11,9 +11,10 @@ GEMM is bracketed by CUDA events on its stream, so flushes are not timed.
               (tera-ops/s; int8 MACs and bf16 FMAs both count 2 ops)
   e2e         the same through the C ABI from pinned HOST buffers: H2D copies
               of A and B, the GEMM, D2H of C, all inside the timed events
-  roofline    the dominant kernel (largest share of step time): the
-              tensor-core kernel of one GEMM, timed alone through the
-              library's profiling events, against the measured bf16 peak
+  roofline    the dominant kernel (largest share of step time): the main
+              kernel of one GEMM (tensor-core, or CUDA-core for tiny M), timed
+              alone through the library's profiling events, against the
+              measured bf16 peak (tensor-bound) or HBM copy bandwidth
   cpu_baseline  the CPU oracle on a bounded sample (whole rows of C) of the
               same GEMMs, on this host's cores
 
@@ -241,19 +242,30 @@ def run_ours(args, rank, world, dev):
 
     peaks, peak_src = load_peaks()
     bf16_peak = float(peaks.get("bf16_tflops", FALLBACK["bf16_tflops"]))
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK["hbm_gbs"]))
     per = []
     for i, c in enumerate(cases):
         ms = statistics.median(per_gemm_ms[i])
         kms = statistics.median(per_kern_ms[i])
         tops = c.g.flops / (ms * 1e-3) / 1e12
-        per.append({"gemm": c.g.name, "ms": round(ms, 5), "tc_kernel_ms": round(kms, 5),
-                    "tops": round(tops, 2), "frac_of_bf16_peak": round(tops / bf16_peak, 4),
-                    "best_ms": round(min(per_gemm_ms[i]), 5)})
-    # dominant kernel: the tensor-core kernel of the GEMM with the largest time
+        gbps = compulsory_bytes(c.g) / (ms * 1e-3) / 1e9
+        per.append({"gemm": c.g.name, "bound": bound_of(c.g, bf16_peak, hbm_peak), "ms": round(ms, 5),
+                    "main_kernel_ms": round(kms, 5), "tops": round(tops, 2),
+                    "frac_of_bf16_peak": round(tops / bf16_peak, 4), "gbps": round(gbps, 1),
+                    "frac_of_hbm": round(gbps / hbm_peak, 4), "best_ms": round(min(per_gemm_ms[i]), 5)})
+    # dominant kernel: the main kernel of the GEMM with the largest time
     dom = max(range(len(cases)), key=lambda i: statistics.mean(per_gemm_ms[i]))
     dk_ms = statistics.mean(per_kern_ms[dom])
-    achieved = cases[dom].g.flops / (dk_ms * 1e-3) / 1e12
     traffic = load_traffic(cases[dom].g.name)
+    if bound_of(cases[dom].g, bf16_peak, hbm_peak) == "tensor":
+        roof = {"bound": "tensor", "kernel": f"main kernel of {cases[dom].g.name}",
+                "achieved": round(cases[dom].g.flops / (dk_ms * 1e-3) / 1e12, 2), "peak": bf16_peak,
+                "unit": "TFLOP/s", "traffic": traffic, "peak_source": f"{peak_src} bf16 dense (burst)"}
+    else:
+        roof = {"bound": "hbm", "kernel": f"main kernel of {cases[dom].g.name}",
+                "achieved": round(compulsory_bytes(cases[dom].g) / (dk_ms * 1e-3) / 1e9, 1), "peak": hbm_peak,
+                "unit": "GB/s", "traffic": traffic, "peak_source": f"{peak_src} HBM copy"}
+    roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -269,10 +281,7 @@ def run_ours(args, rank, world, dev):
                    "gemms": [c.g.name for c in cases], "l2": "flushed (512 MiB write) before every timed GEMM",
                    "parallelism": f"replicas x{world}"},
         "per_gemm": per,
-        "roofline": {"bound": "tensor", "kernel": f"gemm_tc_kernel ({cases[dom].g.name})",
-                     "achieved": round(achieved, 2), "peak": bf16_peak, "unit": "TFLOP/s",
-                     "frac": round(achieved / bf16_peak, 4), "traffic": traffic,
-                     "peak_source": f"{peak_src} bf16 dense (burst)"},
+        "roofline": roof,
         "e2e": None if e2e_ms is None else {
             "value": round(world * ops / (e2e_max * 1e-3) / 1e12, 3), "unit": "TOPS",
             "h2d_bytes_per_step": sum(c.h2d for c in cases), "d2h_bytes_per_step": sum(c.d2h for c in cases)},
@@ -293,6 +302,22 @@ def kernel_source_hash() -> str:
         with open(os.path.join(ROOT, "paper_2512_13282_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
+
+
+def compulsory_bytes(g: W.Gemm) -> int:
+    """Bytes a GEMM must move at least once: A, B and C (Eq. 6-8 of the
+    paper's traffic model with whole-matrix reuse)."""
+    e_in = 1 if g.dtype == "int8" else 2
+    e_out = 4 if g.dtype == "int8" else 2
+    return (g.M * g.K + g.K * g.N) * e_in + g.M * g.N * e_out
+
+
+def bound_of(g: W.Gemm, tflops_peak: float, gbs_peak: float) -> str:
+    """'tensor' when the flops take longer than the compulsory bytes at the
+    measured peaks, else 'hbm'."""
+    t_compute = g.flops / (tflops_peak * 1e12)
+    t_memory = compulsory_bytes(g) / (gbs_peak * 1e9)
+    return "tensor" if t_compute >= t_memory else "hbm"
 
 
 def load_traffic(name):

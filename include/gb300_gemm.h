@@ -159,10 +159,11 @@ gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream
 /*
  * Profiling aid.  With both arguments non-NULL (cudaEvent_t handles created
  * by the caller), every following GEMM call records `start_event` on its
- * stream just before launching its tensor-core kernel and `stop_event` just
- * after, so the time between them covers that kernel alone -- not the
- * operand staging or the split-K reduction passes.  Pass NULL, NULL to stop.
- * Process-wide setting; not meant for concurrent callers.
+ * stream just before launching its main kernel (the tensor-core kernel, or
+ * the CUDA-core kernel for very small M) and `stop_event` just after, so the
+ * time between them covers that kernel alone -- not the operand staging or
+ * split-K reduction passes.  Pass NULL, NULL to stop.  Process-wide setting;
+ * not meant for concurrent callers.
  */
 void gemm_profile_events(void *start_event, void *stop_event);
 

@@ -362,8 +362,12 @@ gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const 
     p.ws = d.ws;
     p.tickets = d.tickets;
   }
+  const bool prof = g_prof_start && g_prof_stop;
+  if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
   g_launches.fetch_add(1);
-  return launch_skinny(p, int8, row_b, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+  if (launch_skinny(p, int8, row_b, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  return GEMM_OK;
 }
 
 }  // namespace
