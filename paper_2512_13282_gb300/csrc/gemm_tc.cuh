@@ -56,7 +56,7 @@ struct TcParams {
   int group_m;       // tiles of M per rasterisation group
   void *C;           // bf16 or int32 output, row-major, leading dimension ldc
   int64_t ldc;
-  int c_vec;         // C rows 16-byte aligned: vector stores allowed
+  int c_vec;         // C rows 16-byte aligned (informational; stores check each address)
   void *ws;          // split-K partials, splits x M x N 32-bit words (fp32 or int32)
   uint32_t *err;     // device error word
   uint64_t wait_limit_ns;
@@ -117,14 +117,36 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&v);
 }
 
+// Store `bytes` (a multiple of 16) of a row chunk that lies fully inside
+// the matrix, with the widest stores the chunk's start address allows
+// (16, 8 or 4 bytes): rows of a C whose leading dimension is not a multiple
+// of 16 bytes are still stored without falling back to one store per
+// element.  `w` holds the chunk as 32-bit words.
+template <int NWORDS>
+__device__ __forceinline__ void store_chunk_aligned(void *dst, const uint32_t (&w)[NWORDS]) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(dst);
+  if ((a & 15) == 0) {
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+    for (int i = 0; i < NWORDS / 4; ++i) d[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+  } else if ((a & 7) == 0) {
+    uint2 *d = reinterpret_cast<uint2 *>(dst);
+#pragma unroll
+    for (int i = 0; i < NWORDS / 2; ++i) d[i] = make_uint2(w[2 * i], w[2 * i + 1]);
+  } else {
+    uint32_t *d = reinterpret_cast<uint32_t *>(dst);
+#pragma unroll
+    for (int i = 0; i < NWORDS; ++i) d[i] = w[i];
+  }
+}
+
 // Store W (16 or 32) consecutive 32-bit words of one row (fp32 partials or
-// int32), vectorised when the row is 16-byte aligned and fully inside N.
+// int32); element-wise only where the chunk crosses column N.
 template <int W>
 __device__ __forceinline__ void store_words(uint32_t *dst, int col, int N, bool vec, const uint32_t (&v)[W]) {
-  if (vec && col + W <= N) {
-    uint4 *d = reinterpret_cast<uint4 *>(dst + col);
-#pragma unroll
-    for (int i = 0; i < W / 4; ++i) d[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+  (void)vec;
+  if (col + W <= N) {
+    store_chunk_aligned<W>(dst + col, v);
   } else {
 #pragma unroll
     for (int i = 0; i < W; ++i)
@@ -135,13 +157,12 @@ __device__ __forceinline__ void store_words(uint32_t *dst, int col, int N, bool 
 // Round W fp32 accumulator words to bf16 (nearest even) and store them.
 template <int W>
 __device__ __forceinline__ void store_bf16(uint16_t *dst, int col, int N, bool vec, const uint32_t (&r)[W]) {
+  (void)vec;
   uint32_t h[W / 2];
 #pragma unroll
   for (int i = 0; i < W / 2; ++i) h[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
-  if (vec && col + W <= N) {
-    uint4 *d = reinterpret_cast<uint4 *>(dst + col);
-#pragma unroll
-    for (int i = 0; i < W / 8; ++i) d[i] = make_uint4(h[4 * i], h[4 * i + 1], h[4 * i + 2], h[4 * i + 3]);
+  if (col + W <= N && (reinterpret_cast<uintptr_t>(dst + col) & 3) == 0) {
+    store_chunk_aligned<W / 2>(dst + col, h);
   } else {
 #pragma unroll
     for (int i = 0; i < W; ++i)
