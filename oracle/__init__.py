@@ -77,6 +77,8 @@ def _declare(lib):
     lib.oracle_gemm_bf16_entries.argtypes = [_i64, _i64, _i64, _ptr, _i64, _ptr, _i64, ctypes.c_int,
                                              _ptr, _ptr, _i64, _ptr, _ptr]
     lib.oracle_rne_bf16.argtypes = [_ptr, _ptr, _i64]
+    lib.oracle_requantize.argtypes = [_ptr, _i64, ctypes.c_int, ctypes.c_int, _ptr]
+    lib.oracle_requantize.restype = ctypes.c_int
     for f in (lib.oracle_gemm_s8, lib.oracle_gemm_bf16, lib.oracle_gemm_s8_entries,
               lib.oracle_gemm_bf16_entries):
         f.restype = ctypes.c_int
@@ -182,6 +184,16 @@ def rne_bf16(x, lib=None) -> np.ndarray:
     x = np.ascontiguousarray(x, dtype=np.float64)
     out = np.zeros(x.shape, dtype=np.uint16)
     (lib or _load()).oracle_rne_bf16(_addr(x), _addr(out), x.size)
+    return out
+
+
+def requantize(acc, shift: int, bits: int, lib=None) -> np.ndarray:
+    """Reduced-precision int8 outputs: exact sums divided by 2^shift, rounded
+    to nearest with ties to even, saturated to a signed `bits`-bit range."""
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
+    out = np.zeros(acc.shape, dtype=np.int64)
+    if (lib or _load()).oracle_requantize(_addr(acc), acc.size, int(shift), int(bits), _addr(out)):
+        raise ValueError("oracle_requantize: shift must be 0..62 and bits 8, 16 or 32")
     return out
 
 

@@ -21,6 +21,10 @@
  * mode, nor what happens when int32 overflows.  The readings taken here are:
  *   - int8:  C[i][j] = sum_k A[i][k]*B(k,j) computed exactly in int64; the
  *            caller checks that it fits int32 (it always does for K <= 131071).
+ *   - int8 reduced-precision outputs (Sec. 5.1 mentions int8-int16 and
+ *            int8-int8 "precision reduction" without a rule): the exact sum
+ *            divided by 2^shift, rounded to nearest with ties to even, then
+ *            saturated to the output's range (oracle_requantize).
  *   - bf16:  inputs decoded exactly to double; ref = sum_k a*b and
  *            mag = sum_k |a*b| in double (every product is exact in double);
  *            rne_bf16() rounds a double straight to the nearest bf16, ties to
@@ -192,4 +196,26 @@ static uint16_t rne_bf16_one(double x) {
 
 void oracle_rne_bf16(const double *x, uint16_t *out, int64_t n) {
   for (int64_t t = 0; t < n; ++t) out[t] = rne_bf16_one(x[t]);
+}
+
+/* Reduced-precision int8 outputs: acc / 2^shift rounded to nearest (ties to
+ * even), saturated to [-2^(bits-1), 2^(bits-1) - 1].  shift in [0, 62],
+ * bits in {8, 16, 32}.  Floor division is written out (no shift of negative
+ * numbers): q = floor(acc / 2^shift), r = acc - q * 2^shift in [0, 2^shift). */
+int oracle_requantize(const int64_t *acc, int64_t n, int shift, int bits, int64_t *out) {
+  if (shift < 0 || shift > 62 || (bits != 8 && bits != 16 && bits != 32)) return 1;
+  const int64_t d = (int64_t)1 << shift;
+  const int64_t hi = ((int64_t)1 << (bits - 1)) - 1, lo = -((int64_t)1 << (bits - 1));
+  for (int64_t t = 0; t < n; ++t) {
+    const int64_t a = acc[t];
+    int64_t q = a / d;               /* truncates toward zero */
+    if (a % d != 0 && a < 0) q -= 1; /* floor */
+    const int64_t r = a - q * d;     /* 0 <= r < d */
+    if (shift > 0) {
+      const int64_t half = d / 2;
+      if (r > half || (r == half && (q % 2 != 0))) q += 1;
+    }
+    out[t] = q > hi ? hi : (q < lo ? lo : q);
+  }
+  return 0;
 }

@@ -236,9 +236,26 @@ def pin_entries(lib):
     assert np.array_equal(r, ref.ravel()) and np.array_equal(g, mag.ravel())
 
 
+def pin_requantize(lib):
+    """Shift-round-saturate: hand-worked ties (to even) and saturation, and
+    numpy's round-half-even division plus clipping on random sums."""
+    acc = np.array([5, 7, -5, -7, 6, -6, 1, -1, 3, -3, 0, 40000, -40000, 2**31 - 1, -2**31], np.int64)
+    want1 = np.array([2, 4, -2, -4, 3, -3, 0, 0, 2, -2, 0, 20000, -20000, 2**30, -2**30], np.int64)
+    assert np.array_equal(oracle.requantize(acc, 1, 32, lib=lib), want1)
+    assert np.array_equal(oracle.requantize(acc, 0, 16, lib=lib),
+                          np.clip(acc, -32768, 32767))
+    assert np.array_equal(oracle.requantize(np.array([383, 384, 385, -383, -384, -385], np.int64), 8, 8, lib=lib),
+                          np.array([1, 2, 2, -1, -2, -2], np.int64))  # 1.496, 1.5 -> 2 (even), 1.504
+    rng = np.random.default_rng(90)
+    a = rng.integers(-2**31, 2**31, 5000, dtype=np.int64)
+    for shift, bits in ((3, 8), (7, 16), (13, 16), (20, 8), (31, 32)):
+        want = np.clip(np.round(a / float(2 ** shift)), -(2 ** (bits - 1)), 2 ** (bits - 1) - 1).astype(np.int64)
+        assert np.array_equal(oracle.requantize(a, shift, bits, lib=lib), want)
+
+
 PINS = [pin_golden, pin_k0_k1, pin_dot_closed_forms, pin_identity_permutation, pin_extremes,
         pin_linearity, pin_layout_and_transpose, pin_numpy_int, pin_numpy_float,
-        pin_integer_bf16_exact, pin_rne_vs_torch, pin_rne_double_cases, pin_entries]
+        pin_integer_bf16_exact, pin_rne_vs_torch, pin_rne_double_cases, pin_entries, pin_requantize]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -283,6 +300,9 @@ MUTANTS = {
     "rne_ties_away": ("const double r = rint(ldexp(ax, 7 - E));",
                       "const double r = round(ldexp(ax, 7 - E));"),
     "rne_no_subnormal_clamp": ("if (E < -126) E = -126;", ""),
+    "requant_ties_away": ("if (r > half || (r == half && (q % 2 != 0))) q += 1;",
+                          "if (r >= half) q += 1;"),
+    "requant_no_floor": ("if (a % d != 0 && a < 0) q -= 1; /* floor */", ""),
     "entries_wrong_index": ("s += (int64_t)A[i * lda + k] * (int64_t)B[b_index(k, j, ldb, layout)];",
                             "s += (int64_t)A[j * lda + k] * (int64_t)B[b_index(k, i, ldb, layout)];"),
 }
