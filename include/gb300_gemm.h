@@ -72,6 +72,29 @@ gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K,
                             int32_t *C, int64_t ldc, gemm_stream_t stream);
 
 /*
+ * int8-int16 and int8-int8 (Sec. 5.1, Tables 1-3: int8 GEMMs whose output
+ * precision is reduced to 16 or 8 bits).  The paper gives no rounding rule;
+ * this library's is:
+ *   C[i][j] = saturate_T(round_half_even(S_ij / 2^shift)),
+ * S_ij = sum_k a_ik * b_kj the exact sum of gemm_s8s8_s32, T = int16 or int8
+ * (saturation to [-32768, 32767] or [-128, 127]).  shift = 0 saturates S
+ * directly.
+ *   A, B, b_layout, K limit and errors: as gemm_s8s8_s32.
+ *   C: M x N row-major int16 / int8 (ldc >= N elements), fully overwritten
+ *   in [0,M) x [0,N); any alignment.
+ *   shift: 0 .. 31, else GEMM_ERR_INVALID_ARG.
+ * Bit-exact: the result is a function of the exact sum only.
+ */
+gemm_status_t gemm_s8s8_s16(int64_t M, int64_t N, int64_t K,
+                            const int8_t *A, int64_t lda,
+                            const int8_t *B, int64_t ldb, int b_layout,
+                            int16_t *C, int64_t ldc, int shift, gemm_stream_t stream);
+gemm_status_t gemm_s8s8_s8(int64_t M, int64_t N, int64_t K,
+                           const int8_t *A, int64_t lda,
+                           const int8_t *B, int64_t ldb, int b_layout,
+                           int8_t *C, int64_t ldc, int shift, gemm_stream_t stream);
+
+/*
  * bf16-bf16 (Sec. 5.1, Table 1): C[i][j] = rne_bf16(sum_k a_ik * b_kj) with
  * the sum accumulated in float32 (any order) and rounded once to bf16,
  * nearest-even.  A, B, C are bf16 bit patterns (uint16_t).

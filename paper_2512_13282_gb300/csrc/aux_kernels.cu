@@ -1,6 +1,6 @@
 // aux_kernels.cu -- the memory-bound helpers around the tensor-core kernel:
 // operand staging (int8 -> bf16, re-pitching misaligned bf16), zero fill for
-// K == 0, and the split-K reduction.
+// K == 0, and the split-K reduction (with the int8 path's requantisation).
 #include <cuda_bf16.h>
 
 #include "gemm_internal.h"
@@ -106,15 +106,23 @@ __global__ void splitk_reduce_bf16_kernel(const float *__restrict__ ws, int spli
   }
 }
 
+// Sum the int32 partials; store as int32, or requantised to int16 / int8.
 __global__ void splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int splits, int64_t M,
-                                         int64_t N, int32_t *__restrict__ C, int64_t ldc) {
+                                         int64_t N, void *__restrict__ C, int64_t ldc, int out_bits,
+                                         int shift) {
   const int64_t total = M * N;
+  const int32_t hi = out_bits == 32 ? INT32_MAX : (1 << (out_bits - 1)) - 1, lo = -hi - 1;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
     int32_t s = 0;
     for (int k = 0; k < splits; ++k) s += ws[(int64_t)k * total + t];
     const int64_t r = t / N, c = t - r * N;
-    C[r * ldc + c] = s;
+    if (out_bits == 32)
+      static_cast<int32_t *>(C)[r * ldc + c] = s;
+    else if (out_bits == 16)
+      static_cast<int16_t *>(C)[r * ldc + c] = (int16_t)requantize_s32(s, shift, lo, hi);
+    else
+      static_cast<int8_t *>(C)[r * ldc + c] = (int8_t)requantize_s32(s, shift, lo, hi);
   }
 }
 
@@ -159,7 +167,9 @@ cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int
 cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esize, int sms,
                              cudaStream_t st) {
   const int g = grid_for(M * N, 4, sms);
-  if (esize == 2)
+  if (esize == 1)
+    zero_fill_kernel<uint8_t><<<g, kThreads, 0, st>>>(static_cast<uint8_t *>(C), M, N, ldc);
+  else if (esize == 2)
     zero_fill_kernel<uint16_t><<<g, kThreads, 0, st>>>(static_cast<uint16_t *>(C), M, N, ldc);
   else
     zero_fill_kernel<int32_t><<<g, kThreads, 0, st>>>(static_cast<int32_t *>(C), M, N, ldc);
@@ -172,9 +182,10 @@ cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, in
   return cudaGetLastError();
 }
 
-cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N,
-                                     int32_t *C, int64_t ldc, int sms, cudaStream_t st) {
-  splitk_reduce_s32_kernel<<<grid_for(M * N, 2, sms), kThreads, 0, st>>>(ws, splits, M, N, C, ldc);
+cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N, void *C,
+                                     int64_t ldc, int out_bits, int shift, int sms, cudaStream_t st) {
+  splitk_reduce_s32_kernel<<<grid_for(M * N, 2, sms), kThreads, 0, st>>>(ws, splits, M, N, C, ldc, out_bits,
+                                                                          shift);
   return cudaGetLastError();
 }
 

@@ -256,6 +256,8 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   p.kb_per_split = (int)kb_per;
   p.slab_kb = epi == kEpiS32 ? 1024 / kBK : (int)num_kb;
   p.group_m = 8;
+  p.out_bits = 32;
+  p.out_shift = 0;
   const int64_t units = tiles * splits;
   const int64_t used = units < slots ? units : slots;
   pl.grid = (int)(pair ? 2 * used : used);
@@ -308,8 +310,8 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
   if (p.splits > 1) {
     e = pl.v.epi == kEpiS32
-            ? launch_splitk_reduce_s32(static_cast<const int32_t *>(partials), p.splits, p.M, p.N,
-                                       static_cast<int32_t *>(C), ldc, d.sms, st)
+            ? launch_splitk_reduce_s32(static_cast<const int32_t *>(partials), p.splits, p.M, p.N, C, ldc,
+                                       p.out_bits, p.out_shift, d.sms, st)
             : launch_splitk_reduce_bf16(static_cast<const float *>(partials), p.splits, p.M, p.N,
                                         static_cast<uint16_t *>(C), ldc, d.sms, st);
     g_launches.fetch_add(1);
@@ -335,7 +337,7 @@ int skinny_max_m(bool int8) {
 
 gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const void *A, int64_t lda,
                          const void *B, int64_t ldb, bool b_kmajor, void *C, int64_t ldc, bool int8,
-                         cudaStream_t st) {
+                         cudaStream_t st, int out_bits = 32, int out_shift = 0) {
   const bool row_b = !b_kmajor;
   const int64_t strips = ceil_div(N, row_b ? 256 : 32);
   SkinnyParams p{};
@@ -349,6 +351,8 @@ gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const 
   p.M = (int)M;
   p.N = N;
   p.K = K;
+  p.out_bits = out_bits;
+  p.out_shift = out_shift;
   const int esize = int8 ? 1 : 2;
   const uintptr_t bb = reinterpret_cast<uintptr_t>(B);
   if (row_b && int8)
@@ -423,23 +427,35 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
   return run_tc(*d, pl, Au, lda_u, Bu, ldb_u, C, ldc, 2, pl.p.splits > 1 ? ws + L.part_off : nullptr, st);
 }
 
-gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
-                            const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
-                            gemm_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// The int8 GEMM behind gemm_s8s8_s32 (out_bits 32), gemm_s8s8_s16 and
+// gemm_s8s8_s8 (out_bits 16 / 8, right shift `shift`): the exact int32 sum
+// is formed the same way for all three; only the final store differs.
+gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda, const int8_t *B,
+                      int64_t ldb, int b_layout, void *C, int64_t ldc, int out_bits, int shift,
+                      gemm_stream_t stream) {
   gemm_status_t s = check_common(M, N, K, A, lda, B, ldb, b_layout, C, ldc);
-  if (s != GEMM_OK || M == 0 || N == 0) return s;
+  if (s != GEMM_OK) return s;
+  if (shift < 0 || shift > 31) return GEMM_ERR_INVALID_ARG;
+  if (M == 0 || N == 0) return GEMM_OK;
   if (K > kMaxExactK) return GEMM_ERR_UNSUPPORTED;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   DeviceState *d = nullptr;
   if ((s = device_state(&d)) != GEMM_OK) return s;
-  if (K == 0) {
+  const int out_esize = out_bits / 8;
+  if (K == 0) {  // every sum is 0, and 0 requantises to 0
     g_launches.fetch_add(1);
-    return launch_zero_fill(C, M, N, ldc, 4, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+    return launch_zero_fill(C, M, N, ldc, out_esize, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
   }
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
   if (M <= skinny_max_m(true))
-    return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, true, st);
+    return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, true, st, out_bits, shift);
   Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
+  pl.p.out_bits = out_bits;
+  pl.p.out_shift = shift;
   // Stage both operands as bf16 (exact for int8) with 16-byte aligned rows.
   const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
   const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;
@@ -459,7 +475,30 @@ gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K, const int8_t *A, in
   if (launch_s8_to_bf16_pair(S8Job{A, M, K, lda, Ab, lda_p}, S8Job{B, b_rows, b_cols, ldb, Bb, ldb_p}, d->sms,
                              st) != cudaSuccess)
     return GEMM_ERR_CUDA;
-  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, pl.p.splits > 1 ? ws + L.part_off : nullptr, st);
+  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, out_esize, pl.p.splits > 1 ? ws + L.part_off : nullptr,
+                st);
+}
+
+}  // namespace
+
+extern "C" {
+
+gemm_status_t gemm_s8s8_s32(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
+                            const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
+                            gemm_stream_t stream) {
+  return s8_gemm(M, N, K, A, lda, B, ldb, b_layout, C, ldc, 32, 0, stream);
+}
+
+gemm_status_t gemm_s8s8_s16(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
+                            const int8_t *B, int64_t ldb, int b_layout, int16_t *C, int64_t ldc, int shift,
+                            gemm_stream_t stream) {
+  return s8_gemm(M, N, K, A, lda, B, ldb, b_layout, C, ldc, 16, shift, stream);
+}
+
+gemm_status_t gemm_s8s8_s8(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
+                           const int8_t *B, int64_t ldb, int b_layout, int8_t *C, int64_t ldc, int shift,
+                           gemm_stream_t stream) {
+  return s8_gemm(M, N, K, A, lda, B, ldb, b_layout, C, ldc, 8, shift, stream);
 }
 
 const char *gemm_status_string(gemm_status_t status) {

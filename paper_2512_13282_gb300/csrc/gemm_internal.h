@@ -48,15 +48,16 @@ cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int
 // One-thread kernel whose bounded mbarrier wait is made to expire
 // (failure-detection self-test).
 cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStream_t st);
-// Fill an M x N block of 16- or 32-bit elements with zero.
+// Fill an M x N block of 8-, 16- or 32-bit elements with zero.
 cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esize, int sms,
                              cudaStream_t st);
 // Split-K reduction: C = round(sum over splits of ws[s]) (fp32 -> bf16 RNE)
-// or C = sum of int32 partials.
+// or C = sum of int32 partials, stored as int32 (out_bits 32) or
+// requantised to out_bits = 16 / 8 with right shift `shift`.
 cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, int64_t N,
                                       uint16_t *C, int64_t ldc, int sms, cudaStream_t st);
-cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N,
-                                     int32_t *C, int64_t ldc, int sms, cudaStream_t st);
+cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N, void *C,
+                                     int64_t ldc, int out_bits, int shift, int sms, cudaStream_t st);
 
 // Argument checks of the int8 entry points (no CUDA calls).
 gemm_status_t validate_s8(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,
@@ -83,6 +84,8 @@ struct SkinnyParams {
   int b_vec;           // B rows allow 16-byte (8-byte for row-major int8) loads
   void *ws;            // ks x M x N 32-bit partials (ks > 1)
   uint32_t *tickets;   // one zeroed counter per column strip (ks > 1)
+  int out_bits;        // int8: 32 (int32 C), 16 or 8 (requantised C)
+  int out_shift;       // int8 with out_bits < 32: right shift, 0..31
 };
 void skinny_split(int64_t K, int64_t strips, int sms, int m_rows, int esize, int *kb, int *ks);
 cudaError_t launch_skinny(const SkinnyParams &p, bool int8, bool row_b, cudaStream_t st);

@@ -41,6 +41,21 @@ __device__ __forceinline__ uint32_t *partial_ptr(const SkinnyParams &p, int slic
 // the final result when ks == 1, else as partials with a last-block sum.
 // `vals` is this block's (already warp-combined) M x cols result in shared
 // memory, row stride `ld` words.
+// One int8-path result: int32, or requantised to int16 / int8.
+__device__ __forceinline__ void store_s8_out(const SkinnyParams &p, int m, int64_t n, int32_t s) {
+  const int64_t at = m * p.ldc + n;
+  if (p.out_bits == 32) {
+    reinterpret_cast<int32_t *>(p.C)[at] = s;
+  } else {
+    const int32_t hi = (1 << (p.out_bits - 1)) - 1, lo = -hi - 1;
+    const int32_t q = requantize_s32(s, p.out_shift, lo, hi);
+    if (p.out_bits == 16)
+      reinterpret_cast<int16_t *>(p.C)[at] = (int16_t)q;
+    else
+      reinterpret_cast<int8_t *>(p.C)[at] = (int8_t)q;
+  }
+}
+
 template <bool INT8>
 __device__ void finish_block(const SkinnyParams &p, const uint32_t *vals, int ld, int64_t n0, int cols,
                              uint32_t *ticket_smem) {
@@ -50,7 +65,7 @@ __device__ void finish_block(const SkinnyParams &p, const uint32_t *vals, int ld
       const int m = t / cols, c = t - m * cols;
       const int64_t n = n0 + c;
       if (INT8) {
-        reinterpret_cast<int32_t *>(p.C)[m * p.ldc + n] = (int32_t)vals[m * ld + c];
+        store_s8_out(p, m, n, (int32_t)vals[m * ld + c]);
       } else {
         __nv_bfloat16 h = __float2bfloat16_rn(__uint_as_float(vals[m * ld + c]));
         reinterpret_cast<uint16_t *>(p.C)[m * p.ldc + n] = *reinterpret_cast<uint16_t *>(&h);
@@ -76,7 +91,7 @@ __device__ void finish_block(const SkinnyParams &p, const uint32_t *vals, int ld
     if (INT8) {
       int32_t s = 0;
       for (int k = 0; k < p.ks; ++k) s += (int32_t)__ldcg(partial_ptr(p, k, m, n));
-      reinterpret_cast<int32_t *>(p.C)[m * p.ldc + n] = s;
+      store_s8_out(p, m, n, s);
     } else {
       float s = 0.f;
       for (int k = 0; k < p.ks; ++k) s += __uint_as_float(__ldcg(partial_ptr(p, k, m, n)));

@@ -60,6 +60,8 @@ struct TcParams {
   void *ws;          // split-K partials, splits x M x N 32-bit words (fp32 or int32)
   uint32_t *err;     // device error word
   uint64_t wait_limit_ns;
+  int out_bits;      // int8 path: 32 (exact int32 C), 16 or 8 (requantised C)
+  int out_shift;     // int8 path with out_bits < 32: right shift, 0..31
 };
 
 __host__ __device__ constexpr uint32_t pow2_at_least(uint32_t x) {
@@ -117,6 +119,20 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&v);
 }
 
+// Reduced-precision int8 outputs (Sec. 5.1 reduces int8 GEMM outputs to 16
+// and 8 bits): the exact sum divided by 2^shift, rounded to nearest with
+// ties to even, saturated to [lo, hi].  shift is 0..31; a >> shift is the
+// floor (arithmetic shift) and r the non-negative remainder.
+__host__ __device__ __forceinline__ int32_t requantize_s32(int32_t a, int shift, int32_t lo, int32_t hi) {
+  int32_t q = a >> shift;
+  if (shift > 0) {
+    const uint32_t r = static_cast<uint32_t>(a) & ((1u << shift) - 1u);
+    const uint32_t half = 1u << (shift - 1);
+    q += (r > half || (r == half && (q & 1))) ? 1 : 0;  // |q| < 2^30 here: no overflow
+  }
+  return q < lo ? lo : (q > hi ? hi : q);
+}
+
 // Store `bytes` (a multiple of 16) of a row chunk that lies fully inside
 // the matrix, with the widest stores the chunk's start address allows
 // (16, 8 or 4 bytes): rows of a C whose leading dimension is not a multiple
@@ -167,6 +183,51 @@ __device__ __forceinline__ void store_bf16(uint16_t *dst, int col, int N, bool v
 #pragma unroll
     for (int i = 0; i < W; ++i)
       if (col + i < N) dst[col + i] = static_cast<uint16_t>(h[i >> 1] >> (16 * (i & 1)));
+  }
+}
+
+// Store W (16 or 32) int32 results of row `row`, columns [col, col + W)
+// clipped at N, into C: as int32, or requantised to int16 / int8 and packed
+// into 32-bit words (per element where the chunk crosses N or the address
+// is not 4-byte aligned).
+template <int W>
+__device__ __forceinline__ void store_s8_result(const TcParams &p, int64_t row, int col, const uint32_t (&v)[W]) {
+  if (p.out_bits == 32) {
+    store_words<W>(reinterpret_cast<uint32_t *>(p.C) + row * p.ldc, col, p.N, true, v);
+    return;
+  }
+  const int32_t hi = (1 << (p.out_bits - 1)) - 1, lo = -hi - 1;
+  int32_t q[W];
+#pragma unroll
+  for (int i = 0; i < W; ++i) q[i] = requantize_s32(static_cast<int32_t>(v[i]), p.out_shift, lo, hi);
+  const bool full = col + W <= p.N;
+  if (p.out_bits == 16) {
+    int16_t *dst = reinterpret_cast<int16_t *>(p.C) + row * p.ldc + col;
+    if (full && (reinterpret_cast<uintptr_t>(dst) & 3) == 0) {
+      uint32_t h[W / 2];
+#pragma unroll
+      for (int i = 0; i < W / 2; ++i)
+        h[i] = (static_cast<uint32_t>(q[2 * i]) & 0xFFFFu) | (static_cast<uint32_t>(q[2 * i + 1]) << 16);
+      store_chunk_aligned<W / 2>(dst, h);
+    } else {
+#pragma unroll
+      for (int i = 0; i < W; ++i)
+        if (col + i < p.N) dst[i] = static_cast<int16_t>(q[i]);
+    }
+  } else {
+    int8_t *dst = reinterpret_cast<int8_t *>(p.C) + row * p.ldc + col;
+    if (full && (reinterpret_cast<uintptr_t>(dst) & 3) == 0) {
+      uint32_t h[W / 4];
+#pragma unroll
+      for (int i = 0; i < W / 4; ++i)
+        h[i] = (static_cast<uint32_t>(q[4 * i]) & 0xFFu) | ((static_cast<uint32_t>(q[4 * i + 1]) & 0xFFu) << 8) |
+               ((static_cast<uint32_t>(q[4 * i + 2]) & 0xFFu) << 16) | (static_cast<uint32_t>(q[4 * i + 3]) << 24);
+      store_chunk_aligned<W / 4>(dst, h);
+    } else {
+#pragma unroll
+      for (int i = 0; i < W; ++i)
+        if (col + i < p.N) dst[i] = static_cast<int8_t>(q[i]);
+    }
   }
 }
 
@@ -358,22 +419,28 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
         }
         if (!ok) break;
         if (row_ok) {
-          uint32_t *dst = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
-                                : reinterpret_cast<uint32_t *>(p.C) + row * p.ldc;
-          const bool vec = split ? ws_vec : (p.c_vec != 0);
+          // split-K partials stay int32; the reduction requantises
+          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                                 : nullptr;
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
-            store_words<32>(dst, col0 + c * 32, p.N, vec, v);
+            if (split)
+              store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, v);
+            else
+              store_s8_result<32>(p, row, col0 + c * 32, v);
           }
           if constexpr (CPT % 32 != 0) {
             constexpr int kTail = (CPT / 32) * 32;
             uint32_t v[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
-            store_words<16>(dst, col0 + kTail, p.N, vec, v);
+            if (split)
+              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+            else
+              store_s8_result<16>(p, row, col0 + kTail, v);
           }
         }
       } else {

@@ -302,22 +302,28 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
         }
         if (!ok) break;
         if (row_ok) {
-          uint32_t *dst = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
-                                : reinterpret_cast<uint32_t *>(p.C) + row * p.ldc;
-          const bool vec = split ? ws_vec : (p.c_vec != 0);
+          // split-K partials stay int32; the reduction requantises
+          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                                 : nullptr;
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
-            store_words<32>(dst, col0 + c * 32, p.N, vec, v);
+            if (split)
+              store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, v);
+            else
+              store_s8_result<32>(p, row, col0 + c * 32, v);
           }
           if constexpr (CPT % 32 != 0) {
             constexpr int kTail = (CPT / 32) * 32;
             uint32_t v[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
-            store_words<16>(dst, col0 + kTail, p.N, vec, v);
+            if (split)
+              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+            else
+              store_s8_result<16>(p, row, col0 + kTail, v);
           }
         }
       } else {

@@ -53,6 +53,10 @@ def library():
             f = getattr(lib, name)
             f.argtypes = [i64, i64, i64, vp, i64, vp, i64, ci, vp, i64, vp]
             f.restype = ci
+        for name in ("gemm_s8s8_s16", "gemm_s8s8_s8"):
+            f = getattr(lib, name)
+            f.argtypes = [i64, i64, i64, vp, i64, vp, i64, ci, vp, i64, ci, vp]
+            f.restype = ci
         lib.gemm_status_string.argtypes = [ci]
         lib.gemm_status_string.restype = ctypes.c_char_p
         lib.gemm_device_status.argtypes = []
@@ -90,6 +94,18 @@ def gemm_s8s8_s32(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int
     """C (int32, M x N) = A (int8, M x K) . B (int8, K x N), exact."""
     return int(library().gemm_s8s8_s32(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
                                        _ptr(C), ldc, _stream(stream)))
+
+
+def gemm_s8s8_s16(M, N, K, A, lda, B, ldb, b_layout, C, ldc, shift, stream=None) -> int:
+    """C (int16) = saturate(round_half_even((A . B) / 2^shift)), A, B int8."""
+    return int(library().gemm_s8s8_s16(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
+                                       _ptr(C), ldc, int(shift), _stream(stream)))
+
+
+def gemm_s8s8_s8(M, N, K, A, lda, B, ldb, b_layout, C, ldc, shift, stream=None) -> int:
+    """C (int8) = saturate(round_half_even((A . B) / 2^shift)), A, B int8."""
+    return int(library().gemm_s8s8_s8(M, N, K, _ptr(A), lda, _ptr(B), ldb, int(b_layout),
+                                      _ptr(C), ldc, int(shift), _stream(stream)))
 
 
 def gemm_s8s8_s32_noalloc(M, N, K, A, lda, B, ldb, b_layout, C, ldc, stream=None) -> int:

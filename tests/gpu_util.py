@@ -29,10 +29,16 @@ def to_device(a: np.ndarray, ld: int = None, offset: int = 0):
     return buf, buf.data_ptr() + offset * buf.element_size(), ld
 
 
+SENTINEL_S16 = 0x5A5A                 # guard values of int16 / int8 outputs
+SENTINEL_S8 = 0x5A
+
+
 def run(dtype, A, B, layout, lda=None, ldb=None, ldc=None, a_off=0, b_off=0, c_off=0,
-        stream=None, expect=G.GEMM_OK):
-    """Run one GEMM through the C ABI.  Returns C (numpy int32 or uint16
-    bit patterns) after checking the guard region of C."""
+        stream=None, expect=G.GEMM_OK, shift=0):
+    """Run one GEMM through the C ABI.  dtype "int8" (int32 C), "s16" / "s8"
+    (int8 operands, requantised int16 / int8 C with right shift `shift`) or
+    "bf16".  Returns C (numpy int32, int16, int8 or uint16 bit patterns) after
+    checking the guard region of C."""
     M, K = A.shape
     N = B.shape[1] if layout == G.GEMM_B_ROW_MAJOR_KxN else B.shape[0]
     # keep the buffers referenced until the GEMM has finished: a dropped
@@ -44,6 +50,13 @@ def run(dtype, A, B, layout, lda=None, ldb=None, ldc=None, a_off=0, b_off=0, c_o
     if dtype == "int8":
         cbuf = torch.full((c_off + (M + 2) * ldc + 16,), SENTINEL32, dtype=torch.int32, device="cuda")
         fn, sent = G.gemm_s8s8_s32, SENTINEL32
+    elif dtype in ("s16", "s8"):
+        tdt, sent = (torch.int16, SENTINEL_S16) if dtype == "s16" else (torch.int8, SENTINEL_S8)
+        cbuf = torch.full((c_off + (M + 2) * ldc + 16,), sent, dtype=tdt, device="cuda")
+        g = G.gemm_s8s8_s16 if dtype == "s16" else G.gemm_s8s8_s8
+
+        def fn(M, N, K, pa, lda, pb, ldb, layout, pc, ldc, stream):
+            return g(M, N, K, pa, lda, pb, ldb, layout, pc, ldc, shift, stream)
     else:
         cbuf = torch.full((c_off + (M + 2) * ldc + 16,), SENTINEL16, dtype=torch.int16, device="cuda")
         fn, sent = G.gemm_bf16_f32acc_bf16, SENTINEL16

@@ -68,6 +68,17 @@ def test_empty_problems_are_noops(lib, fn):
     assert fn(5, 0, 7, 0, 7, 0, 1, 0, 0, 1, stream=0) == G.GEMM_OK
 
 
+@pytest.mark.parametrize("fn", [G.gemm_s8s8_s16, G.gemm_s8s8_s8])
+def test_requantised_outputs_argument_checks_on_host(lib, fn):
+    p = 0x1000
+    for shift in (-1, 32, 100):
+        assert fn(4, 4, 4, p, 4, p, 4, 0, p, 4, shift, stream=0) == G.GEMM_ERR_INVALID_ARG
+    assert fn(4, 5, 4, p, 4, p, 5, 0, p, 4, 3, stream=0) == G.GEMM_ERR_INVALID_ARG  # ldc < N
+    assert fn(4, 4, 4, p, 4, p, 4, 0, 0, 4, 3, stream=0) == G.GEMM_ERR_INVALID_ARG  # null C
+    assert fn(0, 5, 7, 0, 7, 0, 5, 0, 0, 5, 31, stream=0) == G.GEMM_OK
+    assert fn(2, 2, 131072, p, 131072, p, 2, 0, p, 2, 0, stream=0) == G.GEMM_ERR_UNSUPPORTED
+
+
 def test_int8_k_limit_on_host(lib):
     p = 0x1000
     assert G.gemm_s8s8_s32(2, 2, 131072, p, 131072, p, 2, 0, p, 2, stream=0) == G.GEMM_ERR_UNSUPPORTED
