@@ -123,6 +123,15 @@ class GemmCase:
             ha, hb = torch.from_numpy(A), torch.from_numpy(B)
             self.C = torch.empty((g.M, g.N), dtype=torch.int32, device=dev)
             self.fn = G.gemm_s8s8_s32
+        elif g.int8_in:  # int8-int16 / int8-int8: requantised outputs
+            ha, hb = torch.from_numpy(A), torch.from_numpy(B)
+            s16 = g.dtype == "int8_int16"
+            self.C = torch.empty((g.M, g.N), dtype=torch.int16 if s16 else torch.int8, device=dev)
+            narrow = G.gemm_s8s8_s16 if s16 else G.gemm_s8s8_s8
+
+            def fn(M, N, K, A_, lda, B_, ldb, layout, C_, ldc, stream):
+                return narrow(M, N, K, A_, lda, B_, ldb, layout, C_, ldc, g.shift, stream)
+            self.fn = fn
         else:
             ha, hb = torch.from_numpy(A.view(np.int16)), torch.from_numpy(B.view(np.int16))
             self.C = torch.empty((g.M, g.N), dtype=torch.int16, device=dev)
@@ -307,7 +316,7 @@ def run_ours(args, rank, world, dev):
         "metric": METRIC, "value": round(value, 3), "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(gemm_ms, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "int8->int32 and bf16->fp32->bf16", "data": "synthetic (seeded, workloads.py)",
+        "dtype": dtype_desc(wl), "data": "synthetic (seeded, workloads.py)",
         "config": {"workload": wl.name, "description": wl.description,
                    "gemms": [c.g.name for c in cases], "l2": "flushed (512 MiB write) before every timed GEMM",
                    "parallelism": f"replicas x{world}"},
@@ -335,12 +344,24 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
+_DTYPE_DESC = {"int8": "int8->int32", "int8_int16": "int8->int32->int16", "int8_int8": "int8->int32->int8",
+               "bf16": "bf16->fp32->bf16"}
+
+
+def dtype_desc(wl) -> str:
+    """The arithmetic of the workload's GEMMs, e.g. 'int8->int32 and bf16->fp32->bf16'."""
+    seen = []
+    for g in wl.gemms:
+        if _DTYPE_DESC[g.dtype] not in seen:
+            seen.append(_DTYPE_DESC[g.dtype])
+    return " and ".join(seen)
+
+
 def compulsory_bytes(g: W.Gemm) -> int:
     """Bytes a GEMM must move at least once: A, B and C (Eq. 6-8 of the
     paper's traffic model with whole-matrix reuse)."""
-    e_in = 1 if g.dtype == "int8" else 2
-    e_out = 4 if g.dtype == "int8" else 2
-    return (g.M * g.K + g.K * g.N) * e_in + g.M * g.N * e_out
+    e_in = 1 if g.int8_in else 2
+    return (g.M * g.K + g.K * g.N) * e_in + g.M * g.N * g.out_bytes
 
 
 def bound_of(g: W.Gemm, tflops_peak: float, gbs_peak: float) -> str:
@@ -371,8 +392,10 @@ def load_traffic(name):
 def _oracle_rows(g: W.Gemm, A, B, rows):
     import oracle
     As = np.ascontiguousarray(A[:rows])
-    if g.dtype == "int8":
-        oracle.gemm_s8(As, B, g.layout)
+    if g.int8_in:
+        acc = oracle.gemm_s8(As, B, g.layout)
+        if g.dtype != "int8":
+            oracle.requantize(acc, g.shift, 8 * g.out_bytes)
     else:
         oracle.gemm_bf16(As, B, g.layout)
 
@@ -437,7 +460,8 @@ def run_reference(args, rank, world):
         "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t_total / args.steps * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "int8->int64 and bf16->f64 (oracle)", "data": "synthetic (seeded, workloads.py)",
+        "dtype": dtype_desc(wl).replace("int32", "int64").replace("fp32", "f64") + " (oracle)",
+        "data": "synthetic (seeded, workloads.py)",
         "config": {"workload": wl.name, "description": wl.description, "gemms": [g.name for g in wl.gemms]},
         "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": oracle.num_threads(),
                          "kind": "oracle", "sample": sample},

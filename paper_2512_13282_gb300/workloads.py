@@ -38,11 +38,21 @@ class Gemm:
     M: int
     N: int
     K: int
-    dtype: str           # "int8" or "bf16"
+    dtype: str           # "int8" (int32 C), "int8_int16" / "int8_int8" (requantised C) or "bf16"
     layout: int
     seed: int
     a: Dist
     b: Dist
+    shift: int = 0       # right shift of the requantised int8 outputs
+
+    @property
+    def int8_in(self) -> bool:
+        return self.dtype.startswith("int8")
+
+    @property
+    def out_bytes(self) -> int:
+        """Bytes per element of C."""
+        return {"int8": 4, "int8_int16": 2, "int8_int8": 1, "bf16": 2}[self.dtype]
 
     @property
     def flops(self) -> int:
@@ -96,6 +106,12 @@ WORKLOADS = {
         tuple(g for M in (128, 2048)
               for (K, N) in ((4096, 4096), (4096, 11008), (11008, 4096), (4096, 12288))
               for g in _both(M, N, K, B_COL_MAJOR, 3, ib=I8_HALF, bb=BF_002))),
+    "reduced_precision_outputs": Workload(
+        "reduced_precision_outputs",
+        "int8 GEMMs with outputs reduced to int16 (right shift 6) and int8 (right shift 14), "
+        "M=N=K in {4096, 8192}, uniform [-128,127]; A row-major, B column-major (N x K), seed 1",
+        tuple(Gemm(s, s, s, dt, B_COL_MAJOR, 1, I8, I8, sh) for s in (4096, 8192)
+              for dt, sh in (("int8_int16", 6), ("int8_int8", 14)))),
     "irregular_skinny": Workload(
         "irregular_skinny",
         "irregular and skinny shapes (1000,1500,3000), (16,4096,4096), "

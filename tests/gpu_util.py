@@ -35,9 +35,9 @@ SENTINEL_S8 = 0x5A
 
 def run(dtype, A, B, layout, lda=None, ldb=None, ldc=None, a_off=0, b_off=0, c_off=0,
         stream=None, expect=G.GEMM_OK, shift=0):
-    """Run one GEMM through the C ABI.  dtype "int8" (int32 C), "s16" / "s8"
-    (int8 operands, requantised int16 / int8 C with right shift `shift`) or
-    "bf16".  Returns C (numpy int32, int16, int8 or uint16 bit patterns) after
+    """Run one GEMM through the C ABI.  dtype "int8" (int32 C), "int8_int16" /
+    "int8_int8" (int8 operands, requantised int16 / int8 C with right shift
+    `shift`) or "bf16".  Returns C (numpy int32, int16, int8 or uint16 bit patterns) after
     checking the guard region of C."""
     M, K = A.shape
     N = B.shape[1] if layout == G.GEMM_B_ROW_MAJOR_KxN else B.shape[0]
@@ -50,10 +50,11 @@ def run(dtype, A, B, layout, lda=None, ldb=None, ldc=None, a_off=0, b_off=0, c_o
     if dtype == "int8":
         cbuf = torch.full((c_off + (M + 2) * ldc + 16,), SENTINEL32, dtype=torch.int32, device="cuda")
         fn, sent = G.gemm_s8s8_s32, SENTINEL32
-    elif dtype in ("s16", "s8"):
-        tdt, sent = (torch.int16, SENTINEL_S16) if dtype == "s16" else (torch.int8, SENTINEL_S8)
+    elif dtype in ("int8_int16", "int8_int8"):
+        s16 = dtype == "int8_int16"
+        tdt, sent = (torch.int16, SENTINEL_S16) if s16 else (torch.int8, SENTINEL_S8)
         cbuf = torch.full((c_off + (M + 2) * ldc + 16,), sent, dtype=tdt, device="cuda")
-        g = G.gemm_s8s8_s16 if dtype == "s16" else G.gemm_s8s8_s8
+        g = G.gemm_s8s8_s16 if s16 else G.gemm_s8s8_s8
 
         def fn(M, N, K, pa, lda, pb, ldb, layout, pc, ldc, stream):
             return g(M, N, K, pa, lda, pb, ldb, layout, pc, ldc, shift, stream)

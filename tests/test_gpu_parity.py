@@ -215,10 +215,12 @@ def test_full_size_configs_sampled(g):
     """Every GEMM of every workload at full size, in the launch configuration
     the benchmark times: sampled outputs against the oracle, one by one."""
     A, B = W.make_inputs(g)
-    C = U.run(g.dtype, A, B, g.layout)
+    C = U.run(g.dtype, A, B, g.layout, shift=g.shift)
     r, c = _sample_positions(g.M, g.N, seed=g.M + g.N + g.K)
-    if g.dtype == "int8":
+    if g.int8_in:
         want = oracle.gemm_s8_entries(A, B, g.layout, r, c)
+        if g.dtype != "int8":
+            want = oracle.requantize(want, g.shift, 8 * g.out_bytes)
         got = C[r, c].astype(np.int64)
         assert np.array_equal(got, want), f"{np.sum(got != want)} of {r.size} sampled entries differ"
     else:

@@ -15,7 +15,7 @@ from tests import gpu_util as U
 
 pytestmark = pytest.mark.gpu
 ROW, COL = G.GEMM_B_ROW_MAJOR_KxN, G.GEMM_B_COL_MAJOR_NxK
-BITS = {"s16": 16, "s8": 8}
+BITS = {"int8_int16": 16, "int8_int8": 8}
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -49,7 +49,7 @@ def _shift_for(out, K):
 SHAPES = [(1, 1, 1), (5, 7, 3), (129, 257, 65), (300, 520, 200), (1000, 1500, 3000), (257, 129, 2100)]
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M,N,K", SHAPES, ids=[f"{m}x{n}x{k}" for m, n, k in SHAPES])
 def test_requant_parity_shapes(out, layout, M, N, K):
@@ -62,7 +62,7 @@ def test_requant_parity_shapes(out, layout, M, N, K):
         assert (np.abs(want) < lim - 1).mean() > 0.5
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("shift", [0, 1, 7, 13, 31])
 def test_requant_every_shift_class(out, layout, shift):
@@ -71,7 +71,7 @@ def test_requant_every_shift_class(out, layout, shift):
     _check(out, A, B, layout, shift, C)
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("bn", [128, 192, 224, 256])
 @pytest.mark.parametrize("pair", ["0", "1"], ids=["single", "pair"])
@@ -88,7 +88,7 @@ def test_requant_every_tile_width(out, layout, bn, pair, monkeypatch):
     _check(out, A, B, layout, shift, C)
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M,N,K", [(16, 512, 4096), (130, 300, 9000)])
 def test_requant_split_k(out, layout, M, N, K, monkeypatch):
@@ -100,7 +100,7 @@ def test_requant_split_k(out, layout, M, N, K, monkeypatch):
     _check(out, A, B, layout, shift, C)
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M,N,K", [(1, 1000, 777), (3, 4100, 4096), (8, 300, 20000)])
 def test_requant_small_m(out, layout, M, N, K):
@@ -110,7 +110,7 @@ def test_requant_small_m(out, layout, M, N, K):
     _check(out, A, B, layout, shift, C)
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M", [4, 300])
 def test_requant_unaligned_c(out, layout, M):
@@ -122,7 +122,7 @@ def test_requant_unaligned_c(out, layout, M):
     _check(out, A, B, layout, shift, C)
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 def test_requant_extremes_and_ties(out):
     # all -128 with K = 64: every sum is 2^20; shifts 19 and 20 give 2 and 1
     # exactly, 21 a tie (0.5 -> 0), 0 saturates.  A second problem puts
@@ -142,7 +142,7 @@ def test_requant_extremes_and_ties(out):
     assert set(np.unique(want[:, 0] % 2)) == {0}  # ties went to even
 
 
-@pytest.mark.parametrize("out", ["s16", "s8"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 def test_requant_k_zero(out):
     A = np.zeros((7, 0), np.int8)
     B = np.zeros((0, 9), np.int8)
@@ -154,6 +154,6 @@ def test_requant_consistent_with_int32_path():
     # the narrow outputs are the int32 path's results requantised
     A, B = _inputs(700, 1100, 2000, COL, seed=77)
     C32 = U.run("int8", A, B, COL)
-    for out, shift in (("s16", 4), ("s8", 12)):
+    for out, shift in (("int8_int16", 4), ("int8_int8", 12)):
         C = U.run(out, A, B, COL, shift=shift)
         assert np.array_equal(C.astype(np.int64), oracle.requantize(C32.astype(np.int64), shift, BITS[out]))
