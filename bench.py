@@ -470,6 +470,126 @@ def run_reference(args, rank, world):
     }
 
 
+# ------------------------------------------------------- roofline sweep
+
+SWEEP_DTYPES = (("int8", 0), ("int8_int16", 6), ("int8_int8", 14), ("bf16", 0))
+
+
+def run_sweep(args, dev):
+    """Roofline sweep (Sec. 5.2.3): every size of roofline_sweep_sizes() for
+    each output precision and both B layouts.  Operands are the leading
+    M*K / K*N elements of 8192^2 seeded master matrices (tight leading
+    dimensions).  Each GEMM runs once untimed, then `reps` times, each after
+    an L2 flush, between CUDA events; the median is kept.  A few sampled
+    entries of every result are checked against the oracle.  Writes every
+    point to `args.sweep` (JSON) and returns the summary line."""
+    import oracle
+    from paper_2512_13282_gb300 import build as Bld
+    from paper_2512_13282_gb300 import gemm as G
+    Bld.build()
+    G.library()
+    oracle.build()
+    sizes = W.roofline_sweep_sizes(args.sweep_points)
+    big = max(max(m * k, k * n) for m, n, k in sizes)
+    hA8 = W.random_int8((big,), 21).reshape(-1)
+    hB8 = W.random_int8((big,), 22).reshape(-1)
+    hA16 = W.random_bf16((big,), 23).reshape(-1)
+    hB16 = W.random_bf16((big,), 24).reshape(-1)
+    dA8, dB8 = torch.from_numpy(hA8).to(dev), torch.from_numpy(hB8).to(dev)
+    dA16, dB16 = torch.from_numpy(hA16.view(np.int16)).to(dev), torch.from_numpy(hB16.view(np.int16)).to(dev)
+    big_c = max(m * n for m, n, _ in sizes)
+    dC = torch.empty(big_c * 4, dtype=torch.uint8, device=dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    rng = np.random.default_rng(7)
+    peaks, peak_src = load_peaks()
+    bf16_peak = float(peaks.get("bf16_tflops", FALLBACK["bf16_tflops"]))
+    fns = {"int8": G.gemm_s8s8_s32, "bf16": G.gemm_bf16_f32acc_bf16}
+    cdt = {"int8": torch.int32, "int8_int16": torch.int16, "int8_int8": torch.int8, "bf16": torch.int16}
+    uuid = str(getattr(torch.cuda.get_device_properties(dev), "uuid", "") or "")
+    if uuid and not uuid.startswith("GPU-"):
+        uuid = "GPU-" + uuid
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    points, checked, bad = [], 0, 0
+    t_start = time.perf_counter()
+    for dtype, shift in SWEEP_DTYPES:
+        int8 = dtype.startswith("int8")
+        dA, dB = (dA8, dB8) if int8 else (dA16, dB16)
+        hA, hB = (hA8, hB8) if int8 else (hA16, hB16)
+        for layout in (W.B_COL_MAJOR, W.B_ROW_MAJOR):
+            for (M, N, K) in sizes:
+                g = W.Gemm(M, N, K, dtype, layout, 0, W.I8 if int8 else W.BF, W.I8 if int8 else W.BF, shift)
+                ldb = N if layout == W.B_ROW_MAJOR else K
+                C = dC.view(cdt[dtype])[:M * N].view(M, N)
+                if dtype in ("int8_int16", "int8_int8"):
+                    fn = G.gemm_s8s8_s16 if dtype == "int8_int16" else G.gemm_s8s8_s8
+
+                    def launch():
+                        return fn(M, N, K, dA, K, dB, ldb, layout, C, N, shift, None)
+                else:
+                    def launch():
+                        return fns[dtype](M, N, K, dA, K, dB, ldb, layout, C, N, None)
+                if launch() != 0:
+                    raise RuntimeError(f"sweep {g.name}: launch failed")
+                evs = []
+                for _ in range(args.sweep_reps):
+                    flush.fill_(1.0)
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(stream)
+                    launch()
+                    b.record(stream)
+                    evs.append((a, b))
+                r = np.concatenate([rng.integers(0, M, 3), [M - 1]])
+                c = np.concatenate([rng.integers(0, N, 3), [N - 1]])
+                got = C[torch.from_numpy(r).to(dev), torch.from_numpy(c).to(dev)].cpu().numpy()
+                ms = statistics.median(x.elapsed_time(y) for x, y in evs)
+                Ah = hA[:M * K].reshape(M, K)
+                Bh = hB[:K * N].reshape((K, N) if layout == W.B_ROW_MAJOR else (N, K))
+                if int8:
+                    want = oracle.gemm_s8_entries(Ah, Bh, layout, r, c)
+                    if dtype != "int8":
+                        want = oracle.requantize(want, shift, 8 * g.out_bytes)
+                    nbad = int(np.sum(got.astype(np.int64) != want))
+                else:
+                    ref, mag = oracle.gemm_bf16_entries(Ah, Bh, layout, r, c)
+                    nbad = int(np.sum(~oracle.bf16_within_bound(got.view(np.uint16), ref, mag)))
+                checked += r.size
+                bad += nbad
+                tops = g.flops / (ms * 1e-3) / 1e12
+                points.append({"dtype": dtype, "layout": "col" if layout == W.B_COL_MAJOR else "row",
+                               "M": M, "N": N, "K": K, "ms": round(ms, 5), "tops": round(tops, 2),
+                               "ari": round(g.flops / compulsory_bytes(g), 1), "mismatches": nbad})
+    torch.cuda.synchronize()
+    sampler.stop()
+    wall = time.perf_counter() - t_start
+
+    summary = {}
+    for dtype, _ in SWEEP_DTYPES:
+        per = {}
+        for lay in ("col", "row"):
+            v = [p for p in points if p["dtype"] == dtype and p["layout"] == lay]
+            t = np.array([p["tops"] for p in v])
+            hi = np.array([p["tops"] for p in v if p["ari"] > 1000])
+            best = max(v, key=lambda p: p["tops"])
+            per[lay] = {"points": len(v), "mean_tops": round(float(t.mean()), 1),
+                        "median_tops": round(float(np.median(t)), 1), "max_tops": best["tops"],
+                        "max_at": [best["M"], best["N"], best["K"]],
+                        "mean_frac_of_bf16_peak": round(float(t.mean()) / bf16_peak, 4),
+                        "ari_gt_1000": {"points": int(hi.size),
+                                        "mean_tops": round(float(hi.mean()), 1) if hi.size else None,
+                                        "cov": round(float(hi.std() / hi.mean()), 4) if hi.size else None}}
+        per["col_over_row_mean_pct"] = round(100.0 * (per["col"]["mean_tops"] / per["row"]["mean_tops"] - 1), 2)
+        summary[dtype] = per
+    with open(args.sweep, "w") as f:
+        json.dump({"sizes_rule": W.roofline_sweep_sizes.__doc__.split("\n")[0], "points": points}, f)
+    return {"metric": "roofline sweep: TOPS per GEMM size, B column- and row-major", "unit": "TOPS",
+            "sizes_per_layout": len(sizes), "gemms": len(points), "reps": args.sweep_reps,
+            "peak_bf16_tflops": bf16_peak, "peak_source": peak_src, "summary": summary,
+            "parity": {"entries_checked": checked, "mismatches": bad}, "clocks": sampler.summary(),
+            "wall_s": round(wall, 1), "points_file": args.sweep}
+
+
 def select(args) -> W.Workload:
     """The workload, optionally narrowed to the GEMMs named by --gemm."""
     wl = W.WORKLOADS[args.workload]
@@ -494,6 +614,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=30.0)
     ap.add_argument("--cpu-seconds-per-step", type=float, default=6.0)
+    ap.add_argument("--sweep", metavar="OUT.json",
+                    help="run the roofline sweep instead (every point written to OUT.json)")
+    ap.add_argument("--sweep-points", type=int, default=420)
+    ap.add_argument("--sweep-reps", type=int, default=3)
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -509,6 +633,10 @@ def main():
 
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    if args.sweep:
+        if rank == 0:
+            print(json.dumps(run_sweep(args, dev)), flush=True)
+        return
     if world > 1:
         torch.distributed.init_process_group("nccl", device_id=dev)
     line = run_ours(args, rank, world, dev)

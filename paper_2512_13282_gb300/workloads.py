@@ -123,6 +123,26 @@ WORKLOADS = {
 }
 
 
+def roofline_sweep_sizes(points: int = 420, seed: int = 5, step: int = 256, largest: int = 8192):
+    """(M, N, K) triples of the roofline sweep: the paper sweeps more than
+    400 sizes per B layout, each a multiple of the native GEMM size, up to
+    8K, favouring no dimension (Sec. 5.2.3).  Here the native size is 256
+    (the CTA-pair tile); M, N and K are drawn independently as step * j,
+    j in 1 .. largest/step with probability proportional to 1/j (uniform in
+    log size, so small and large arithmetic intensities are both well
+    covered), without repeated triples, from numpy's default_rng(seed)."""
+    rng = np.random.default_rng(seed)
+    j = np.arange(1, largest // step + 1)
+    prob = (1.0 / j) / np.sum(1.0 / j)
+    seen, out = set(), []
+    while len(out) < points:
+        t = tuple(int(step * x) for x in rng.choice(j, 3, p=prob))
+        if t not in seen:
+            seen.add(t)
+            out.append(t)
+    return out
+
+
 def _draw(gen: torch.Generator, rows: int, cols: int, d: Dist) -> np.ndarray:
     if d.kind == "int8":
         t = torch.randint(d.lo, d.hi + 1, (rows, cols), generator=gen, dtype=torch.int8)
