@@ -38,21 +38,30 @@ __device__ __forceinline__ void s8x16_to_bf16x16(const int4 raw, uint4 &lo, uint
   hi = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-constexpr int kS8Chunk = 32;       // int8 elements per thread
-constexpr int kS8Threads = 128;    // threads per block: 4096 columns per block
+constexpr int kS8Chunk = 32;       // int8 elements per work item
+constexpr int kS8Threads = 256;
 
-// blockIdx.z selects the job (A or B); blockIdx.y walks rows (strided by
-// gridDim.y); blockIdx.x covers 4096-column slices of a row; each thread
-// converts 32 consecutive elements.  Aligned full chunks use two 16-byte
-// loads and four 16-byte stores.
-__global__ void __launch_bounds__(kS8Threads) s8_to_bf16_pair_kernel(const S8Job a, const S8Job b) {
-  const S8Job j = blockIdx.z == 0 ? a : b;
-  const int64_t c = ((int64_t)blockIdx.x * kS8Threads + threadIdx.x) * kS8Chunk;
-  if (c >= j.cols) return;
-  const bool full = c + kS8Chunk <= j.cols;
-  for (int64_t r = blockIdx.y; r < j.rows; r += gridDim.y) {
-    const int8_t *src = j.src + r * j.ld_src + c;
-    uint16_t *dst = j.dst + r * j.ld_dst + c;
+// Both matrices as one flat list of work items: item t < items_a is chunk
+// t % cpr_a of row t / cpr_a of A (cpr = chunks per row, 32 elements each),
+// the rest likewise of B.  A grid-stride loop over one resident wave of
+// blocks covers wide and narrow matrices alike.  Aligned full chunks use two
+// 16-byte loads and four 16-byte stores.  The next kernel (the GEMM) may be
+// scheduled at once: it waits for this grid's completion before reading.
+__global__ void __launch_bounds__(kS8Threads)
+    s8_to_bf16_pair_kernel(const S8Job a, const S8Job b, int64_t cpr_a, int64_t cpr_b, int64_t items_a,
+                           int64_t items) {
+  griddep_launch_dependents();
+  for (int64_t t = (int64_t)blockIdx.x * kS8Threads + threadIdx.x; t < items;
+       t += (int64_t)gridDim.x * kS8Threads) {
+    const bool in_a = t < items_a;
+    const int64_t u = in_a ? t : t - items_a;
+    const int64_t cpr = in_a ? cpr_a : cpr_b;
+    const int64_t r = u / cpr;
+    const int64_t c = (u - r * cpr) * kS8Chunk;
+    const int64_t cols = in_a ? a.cols : b.cols;
+    const int8_t *src = (in_a ? a.src : b.src) + r * (in_a ? a.ld_src : b.ld_src) + c;
+    uint16_t *dst = (in_a ? a.dst : b.dst) + r * (in_a ? a.ld_dst : b.ld_dst) + c;
+    const bool full = c + kS8Chunk <= cols;
     if (full && (reinterpret_cast<uintptr_t>(src) & 15) == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
       const int4 r0 = __ldg(reinterpret_cast<const int4 *>(src));
       const int4 r1 = __ldg(reinterpret_cast<const int4 *>(src) + 1);
@@ -65,14 +74,43 @@ __global__ void __launch_bounds__(kS8Threads) s8_to_bf16_pair_kernel(const S8Job
       dv[2] = o2;
       dv[3] = o3;
     } else {
-      const int64_t n = j.cols - c < kS8Chunk ? j.cols - c : kS8Chunk;
+      const int64_t n = cols - c < kS8Chunk ? cols - c : kS8Chunk;
       for (int64_t i = 0; i < n; ++i) dst[i] = (uint16_t)s8_to_bf16_bits(src[i]);
     }
   }
 }
 
+// Dense fast path: both matrices contiguous (leading dimension = columns,
+// source 16-byte aligned), so each is one flat array; thread v converts
+// 16-element vector v (v < va: of A, else of B) with one 16-byte load and
+// two 16-byte stores, over a grid that covers every vector once (measured on
+// GB300 faster than fewer threads looping over several vectors).  A last
+// partial vector (elements % 16) is converted element by element.
+__global__ void __launch_bounds__(kS8Threads)
+    s8_to_bf16_dense_kernel(const S8Job a, const S8Job b, int64_t na, int64_t nb) {
+  griddep_launch_dependents();
+  const int64_t va = (na + 15) / 16, vtot = va + (nb + 15) / 16;
+  const int64_t v = (int64_t)blockIdx.x * kS8Threads + threadIdx.x;
+  if (v >= vtot) return;
+  const bool in_a = v < va;
+  const S8Job &j = in_a ? a : b;
+  const int64_t n = in_a ? na : nb;
+  const int64_t e = (in_a ? v : v - va) * 16;
+  if (e + 16 <= n) {
+    const int4 raw = __ldcs(reinterpret_cast<const int4 *>(j.src + e));
+    uint4 lo, hi;
+    s8x16_to_bf16x16(raw, lo, hi);
+    uint4 *d = reinterpret_cast<uint4 *>(j.dst + e);
+    d[0] = lo;
+    d[1] = hi;
+  } else {
+    for (int64_t i = e; i < n; ++i) j.dst[i] = (uint16_t)s8_to_bf16_bits(j.src[i]);
+  }
+}
+
 __global__ void pack_u16_kernel(const uint16_t *__restrict__ src, int64_t rows, int64_t cols,
                                 int64_t ld_src, uint16_t *__restrict__ dst, int64_t ld_dst) {
+  griddep_launch_dependents();  // the GEMM waits for completion before reading
   const int64_t total = rows * cols;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
@@ -95,6 +133,7 @@ __global__ void zero_fill_kernel(T *C, int64_t M, int64_t N, int64_t ldc) {
 // round once to bf16, nearest even.
 __global__ void splitk_reduce_bf16_kernel(const float *__restrict__ ws, int splits, int64_t M,
                                           int64_t N, uint16_t *__restrict__ C, int64_t ldc) {
+  griddep_wait();  // the partials come from the GEMM launched just before
   const int64_t total = M * N;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
@@ -110,6 +149,7 @@ __global__ void splitk_reduce_bf16_kernel(const float *__restrict__ ws, int spli
 __global__ void splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int splits, int64_t M,
                                          int64_t N, void *__restrict__ C, int64_t ldc, int out_bits,
                                          int shift) {
+  griddep_wait();
   const int64_t total = M * N;
   const int32_t hi = out_bits == 32 ? INT32_MAX : (1 << (out_bits - 1)) - 1, lo = -hi - 1;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
@@ -149,12 +189,32 @@ cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStre
 }
 
 cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cudaStream_t st) {
-  (void)sms;
-  const int64_t per_block = (int64_t)kS8Threads * kS8Chunk;
-  const int64_t cols = a.cols > b.cols ? a.cols : b.cols;
-  const int64_t rows = a.rows > b.rows ? a.rows : b.rows;
-  const dim3 grid((unsigned)((cols + per_block - 1) / per_block), (unsigned)(rows < 65535 ? rows : 65535), 2);
-  s8_to_bf16_pair_kernel<<<grid, kS8Threads, 0, st>>>(a, b);
+  static int blocks_per_sm = 0;  // resident blocks per SM (same on every GB300)
+  if (blocks_per_sm == 0) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, s8_to_bf16_pair_kernel, kS8Threads, 0) != cudaSuccess ||
+        n < 1)
+      n = 4;
+    blocks_per_sm = n;
+  }
+  auto dense = [](const S8Job &j) {
+    return j.ld_src == j.cols && j.ld_dst == j.cols && (reinterpret_cast<uintptr_t>(j.src) & 15) == 0 &&
+           (reinterpret_cast<uintptr_t>(j.dst) & 15) == 0;
+  };
+  if (dense(a) && dense(b)) {
+    const int64_t na = a.rows * a.cols, nb = b.rows * b.cols;
+    const int64_t vecs = (na + 15) / 16 + (nb + 15) / 16;
+    if (vecs == 0) return cudaSuccess;
+    s8_to_bf16_dense_kernel<<<(unsigned)((vecs + kS8Threads - 1) / kS8Threads), kS8Threads, 0, st>>>(a, b, na, nb);
+    return cudaGetLastError();
+  }
+  const int64_t cpr_a = (a.cols + kS8Chunk - 1) / kS8Chunk, cpr_b = (b.cols + kS8Chunk - 1) / kS8Chunk;
+  const int64_t items_a = a.rows * cpr_a, items = items_a + b.rows * cpr_b;
+  if (items == 0) return cudaSuccess;
+  const int64_t want = (items + kS8Threads - 1) / kS8Threads;
+  const int64_t wave = (int64_t)sms * blocks_per_sm;
+  const unsigned grid = (unsigned)(want < wave ? want : wave);
+  s8_to_bf16_pair_kernel<<<grid, kS8Threads, 0, st>>>(a, b, cpr_a, cpr_b, items_a, items);
   return cudaGetLastError();
 }
 
@@ -178,15 +238,14 @@ cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esi
 
 cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, int64_t N,
                                       uint16_t *C, int64_t ldc, int sms, cudaStream_t st) {
-  splitk_reduce_bf16_kernel<<<grid_for(M * N, 2, sms), kThreads, 0, st>>>(ws, splits, M, N, C, ldc);
-  return cudaGetLastError();
+  return launch_ex(splitk_reduce_bf16_kernel, dim3(grid_for(M * N, 2, sms)), dim3(kThreads), 0, st, 1, ws, splits,
+                   M, N, C, ldc);
 }
 
 cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N, void *C,
                                      int64_t ldc, int out_bits, int shift, int sms, cudaStream_t st) {
-  splitk_reduce_s32_kernel<<<grid_for(M * N, 2, sms), kThreads, 0, st>>>(ws, splits, M, N, C, ldc, out_bits,
-                                                                          shift);
-  return cudaGetLastError();
+  return launch_ex(splitk_reduce_s32_kernel, dim3(grid_for(M * N, 2, sms)), dim3(kThreads), 0, st, 1, ws, splits,
+                   M, N, C, ldc, out_bits, shift);
 }
 
 }  // namespace gb300

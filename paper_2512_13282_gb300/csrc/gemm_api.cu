@@ -42,6 +42,15 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::atomic<uint64_t> g_launches{0};
 cudaEvent_t g_prof_start = nullptr, g_prof_stop = nullptr;
 
+}  // namespace
+
+bool gb300::pdl_enabled() {
+  const char *s = std::getenv("GB300_GEMM_PDL");
+  return !(s && std::atoi(s) == 0);
+}
+
+namespace {
+
 uint64_t wait_limit_ns() {
   static uint64_t v = [] {
     const char *s = std::getenv("GB300_GEMM_WAIT_LIMIT_MS");

@@ -5,11 +5,47 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <utility>
 
 #include "gb300_gemm.h"
 #include "gemm_tc.cuh"
 
 namespace gb300 {
+
+// Whether kernels that consume the previous kernel's output (the tcgen05
+// GEMM after operand staging, the split-K reduction after the GEMM) are
+// launched with programmatic stream serialisation, so that their launch and
+// set-up overlap the previous kernel's tail (GB300_GEMM_PDL=0 turns it off).
+bool pdl_enabled();
+
+// cudaLaunchKernelEx with programmatic stream serialisation when
+// pdl_enabled(), plus a cluster dimension when cluster_x > 1.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, int cluster_x,
+                      Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  if (cluster_x > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = (unsigned)cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  if (pdl_enabled()) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
 
 // One compiled variant of the tcgen05 kernel.
 struct TcVariant {

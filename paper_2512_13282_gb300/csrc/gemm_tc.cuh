@@ -283,6 +283,10 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
+  // Everything above only touched this CTA's shared memory, TMEM and the
+  // kernel parameters, and may overlap the previous kernel of the stream;
+  // global memory is touched only after that kernel has completed.
+  griddep_wait();
 
   const int num_units = p.tiles_m * p.tiles_n * p.splits;
   constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
@@ -484,6 +488,7 @@ uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
     }
   }
 
+  griddep_launch_dependents();  // e.g. the split-K reduction may start setting up
   __syncwarp();
   tc_fence_before_sync();
   __syncthreads();

@@ -20,19 +20,8 @@ cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const TcPara
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)grid, 1, 1);  // even: a whole number of pairs
-  cfg.blockDim = dim3(Cfg::kThreads, 1, 1);
-  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, a, b, p);
+  // grid is even: a whole number of pairs
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 2, a, b, p);
 }
 
 }  // namespace gb300

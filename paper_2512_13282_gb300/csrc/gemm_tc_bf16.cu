@@ -19,8 +19,7 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParam
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
-  kern<<<grid, Cfg::kThreads, Cfg::kSmemBytes, st>>>(a, b, p);
-  return cudaGetLastError();
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, p);
 }
 }  // namespace
 

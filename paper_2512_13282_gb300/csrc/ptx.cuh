@@ -85,6 +85,20 @@ __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, u
   return true;
 }
 
+// ----------------------------------------------- programmatic dependent launch
+
+// Blocks until every grid this one depends on has completed and its memory
+// operations are visible.  A no-op for a grid launched without a
+// programmatic dependency.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Lets the next grid of the stream, if it was launched with programmatic
+// stream serialisation, be scheduled before this one finishes (it still
+// waits in griddep_wait for this grid's completion).
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // --------------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void tma_prefetch_desc(const void *tmap) {

@@ -287,3 +287,48 @@ def test_small_m_int8_extremes(monkeypatch):
         B = np.full((K, N) if layout == ROW else (N, K), -128, np.int8)
         C = U.run("int8", A, B, layout)
         assert (C == 2147467264).all()
+
+
+# ------------------------------------------- int8 operand staging variants
+
+STAGING = [(300, 520, 256), (1000, 1500, 3000), (257, 129, 4096), (640, 2048, 784), (2048, 2048, 2048),
+           (200, 300, 775)]
+
+
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("M,N,K", STAGING, ids=[f"{m}x{n}x{k}" for m, n, k in STAGING])
+@pytest.mark.parametrize("pdl", ["1", "0"], ids=["pdl", "nopdl"])
+def test_int8_staging_with_and_without_programmatic_launch(layout, M, N, K, pdl, monkeypatch):
+    """The staging pass (flat vectors for tight operands, per-row chunks
+    otherwise) followed by the GEMM, launched with and without programmatic
+    dependent launch: bit-exact either way."""
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    monkeypatch.setenv("GB300_GEMM_PDL", pdl)
+    A, B = _inputs("int8", M, N, K, layout, seed=M ^ N ^ K)
+    C = U.run("int8", A, B, layout)
+    _check("int8", A, B, layout, C)
+
+
+def test_int8_back_to_back_calls(monkeypatch):
+    """Calls queued back to back on one stream without synchronising (pairs,
+    split-K and its reduction included) share the staging workspace: each
+    GEMM must read its own staged operands, never the next call's."""
+    seq = [(2048, 1024, 4096, COL, "1", None), (512, 512, 512, ROW, "0", None),
+           (130, 700, 8192, COL, "0", "4"), (1024, 2048, 1024, ROW, "1", None), (2048, 1024, 4096, COL, "1", None)]
+    keep = []
+    for M, N, K, layout, pair, splits in seq:
+        monkeypatch.setenv("GB300_GEMM_PAIR", pair)
+        if splits:
+            monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
+        else:
+            monkeypatch.delenv("GB300_GEMM_SPLITS", raising=False)
+        A, B = _inputs("int8", M, N, K, layout, seed=K + M)
+        abuf, pa, lda = U.to_device(A)
+        bbuf, pb, ldb = U.to_device(B)
+        C = torch.empty((M, N), dtype=torch.int32, device="cuda")
+        assert G.gemm_s8s8_s32(M, N, K, pa, lda, pb, ldb, layout, C, N) == G.GEMM_OK
+        keep.append((A, B, layout, abuf, bbuf, C))
+    torch.cuda.synchronize()
+    assert G.gemm_device_status() == G.GEMM_OK
+    for A, B, layout, _, _, C in keep:
+        _check("int8", A, B, layout, C.cpu().numpy())
