@@ -3,6 +3,8 @@
 // K == 0, and the split-K reduction (with the int8 path's requantisation).
 #include <cuda_bf16.h>
 
+#include <cstring>
+
 #include "gemm_internal.h"
 
 namespace gb300 {
@@ -38,45 +40,49 @@ __device__ __forceinline__ void s8x16_to_bf16x16(const int4 raw, uint4 &lo, uint
   hi = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-constexpr int kS8Chunk = 32;       // int8 elements per work item
 constexpr int kS8Threads = 256;
 
-// Both matrices as one flat list of work items: item t < items_a is chunk
-// t % cpr_a of row t / cpr_a of A (cpr = chunks per row, 32 elements each),
-// the rest likewise of B.  A grid-stride loop over one resident wave of
-// blocks covers wide and narrow matrices alike.  Aligned full chunks use two
-// 16-byte loads and four 16-byte stores.  The next kernel (the GEMM) may be
-// scheduled at once: it waits for this grid's completion before reading.
+// General path (any alignment, any leading dimension): both matrices as one
+// flat list of 4-element row pieces -- piece t < items_a is piece t % cpr_a
+// of row t / cpr_a of A (cpr = pieces per row), the rest likewise of B.
+// Consecutive threads take consecutive pieces of a row, so a warp reads 128
+// contiguous bytes (one 4-byte load per thread where the row allows it, four
+// byte loads otherwise) and writes 256 contiguous bytes (one 8-byte store:
+// staged rows start 16-byte aligned and pieces are 8 bytes apart).
 __global__ void __launch_bounds__(kS8Threads)
-    s8_to_bf16_pair_kernel(const S8Job a, const S8Job b, int64_t cpr_a, int64_t cpr_b, int64_t items_a,
-                           int64_t items) {
+    s8_to_bf16_pair_kernel(const S8Job a, const S8Job b, uint32_t cpr_a, uint32_t cpr_b, uint64_t items_a,
+                           uint64_t items) {
   griddep_launch_dependents();
-  for (int64_t t = (int64_t)blockIdx.x * kS8Threads + threadIdx.x; t < items;
-       t += (int64_t)gridDim.x * kS8Threads) {
-    const bool in_a = t < items_a;
-    const int64_t u = in_a ? t : t - items_a;
-    const int64_t cpr = in_a ? cpr_a : cpr_b;
-    const int64_t r = u / cpr;
-    const int64_t c = (u - r * cpr) * kS8Chunk;
-    const int64_t cols = in_a ? a.cols : b.cols;
-    const int8_t *src = (in_a ? a.src : b.src) + r * (in_a ? a.ld_src : b.ld_src) + c;
-    uint16_t *dst = (in_a ? a.dst : b.dst) + r * (in_a ? a.ld_dst : b.ld_dst) + c;
-    const bool full = c + kS8Chunk <= cols;
-    if (full && (reinterpret_cast<uintptr_t>(src) & 15) == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
-      const int4 r0 = __ldg(reinterpret_cast<const int4 *>(src));
-      const int4 r1 = __ldg(reinterpret_cast<const int4 *>(src) + 1);
-      uint4 o0, o1, o2, o3;
-      s8x16_to_bf16x16(r0, o0, o1);
-      s8x16_to_bf16x16(r1, o2, o3);
-      uint4 *dv = reinterpret_cast<uint4 *>(dst);
-      dv[0] = o0;
-      dv[1] = o1;
-      dv[2] = o2;
-      dv[3] = o3;
+  const uint64_t t = (uint64_t)blockIdx.x * kS8Threads + threadIdx.x;
+  if (t >= items) return;
+  const bool in_a = t < items_a;
+  const S8Job &j = in_a ? a : b;
+  const uint64_t u = in_a ? t : t - items_a;
+  const uint32_t cpr = in_a ? cpr_a : cpr_b;
+  uint64_t r, q;
+  if (u <= 0xFFFFFFFFull) {
+    r = (uint32_t)u / cpr;
+    q = (uint32_t)u - (uint32_t)r * cpr;
+  } else {
+    r = u / cpr;
+    q = u - r * cpr;
+  }
+  const int64_t c = (int64_t)q * 4;
+  const int8_t *src = j.src + (int64_t)r * j.ld_src + c;
+  uint16_t *dst = j.dst + (int64_t)r * j.ld_dst + c;
+  if (c + 4 <= j.cols) {
+    uint32_t w;
+    if ((reinterpret_cast<uintptr_t>(src) & 3) == 0) {
+      w = __ldcs(reinterpret_cast<const unsigned int *>(src));
     } else {
-      const int64_t n = cols - c < kS8Chunk ? cols - c : kS8Chunk;
-      for (int64_t i = 0; i < n; ++i) dst[i] = (uint16_t)s8_to_bf16_bits(src[i]);
+      w = (uint32_t)(uint8_t)src[0] | ((uint32_t)(uint8_t)src[1] << 8) | ((uint32_t)(uint8_t)src[2] << 16) |
+          ((uint32_t)(uint8_t)src[3] << 24);
     }
+    const uint32_t lo = s8_to_bf16_bits((int8_t)(w & 0xFF)) | (s8_to_bf16_bits((int8_t)((w >> 8) & 0xFF)) << 16);
+    const uint32_t hi = s8_to_bf16_bits((int8_t)((w >> 16) & 0xFF)) | (s8_to_bf16_bits((int8_t)(w >> 24)) << 16);
+    *reinterpret_cast<uint2 *>(dst) = make_uint2(lo, hi);
+  } else {
+    for (int64_t i = 0; c + i < j.cols; ++i) dst[i] = (uint16_t)s8_to_bf16_bits(src[i]);
   }
 }
 
@@ -108,14 +114,42 @@ __global__ void __launch_bounds__(kS8Threads)
   }
 }
 
-__global__ void pack_u16_kernel(const uint16_t *__restrict__ src, int64_t rows, int64_t cols,
-                                int64_t ld_src, uint16_t *__restrict__ dst, int64_t ld_dst) {
+// Re-pitch of a bf16 matrix into a buffer whose rows start 16-byte aligned:
+// thread t copies 4-element piece t % cpr of row t / cpr (one 8-byte load
+// where the source row allows it, else two 4-byte or four 2-byte loads; one
+// 8-byte store).
+__global__ void __launch_bounds__(kS8Threads)
+    pack_u16_kernel(const uint16_t *__restrict__ src, int64_t cols, int64_t ld_src, uint16_t *__restrict__ dst,
+                    int64_t ld_dst, uint32_t cpr, uint64_t items) {
   griddep_launch_dependents();  // the GEMM waits for completion before reading
-  const int64_t total = rows * cols;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = t / cols, c = t - r * cols;
-    dst[r * ld_dst + c] = src[r * ld_src + c];
+  const uint64_t t = (uint64_t)blockIdx.x * kS8Threads + threadIdx.x;
+  if (t >= items) return;
+  uint64_t r, q;
+  if (t <= 0xFFFFFFFFull) {
+    r = (uint32_t)t / cpr;
+    q = (uint32_t)t - (uint32_t)r * cpr;
+  } else {
+    r = t / cpr;
+    q = t - r * cpr;
+  }
+  const int64_t c = (int64_t)q * 4;
+  const uint16_t *s = src + (int64_t)r * ld_src + c;
+  uint16_t *d = dst + (int64_t)r * ld_dst + c;
+  if (c + 4 <= cols) {
+    const uintptr_t al = reinterpret_cast<uintptr_t>(s);
+    uint2 v;
+    if ((al & 7) == 0) {
+      v = __ldcs(reinterpret_cast<const uint2 *>(s));
+    } else if ((al & 3) == 0) {
+      v.x = __ldcs(reinterpret_cast<const unsigned int *>(s));
+      v.y = __ldcs(reinterpret_cast<const unsigned int *>(s) + 1);
+    } else {
+      v.x = (uint32_t)s[0] | ((uint32_t)s[1] << 16);
+      v.y = (uint32_t)s[2] | ((uint32_t)s[3] << 16);
+    }
+    *reinterpret_cast<uint2 *>(d) = v;
+  } else {
+    for (int64_t i = 0; c + i < cols; ++i) d[i] = s[i];
   }
 }
 
@@ -129,40 +163,109 @@ __global__ void zero_fill_kernel(T *C, int64_t M, int64_t N, int64_t ldc) {
   }
 }
 
-// Sum the fp32 partials of all splits (fixed order: split 0, 1, ...), then
-// round once to bf16, nearest even.
-__global__ void splitk_reduce_bf16_kernel(const float *__restrict__ ws, int splits, int64_t M,
-                                          int64_t N, uint16_t *__restrict__ C, int64_t ldc) {
-  griddep_wait();  // the partials come from the GEMM launched just before
-  const int64_t total = M * N;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    float s = 0.f;
-    for (int k = 0; k < splits; ++k) s += ws[(int64_t)k * total + t];
-    const int64_t r = t / N, c = t - r * N;
-    __nv_bfloat16 h = __float2bfloat16_rn(s);
-    C[r * ldc + c] = *reinterpret_cast<uint16_t *>(&h);
+// Split-K reduction: thread t sums 4-element piece t % cpr of row t / cpr
+// over the splits in a fixed order (split 0, 1, ...), with 16-byte partial
+// loads when N is a multiple of 4, and stores the piece with one store where
+// C's address allows it.
+struct Piece {
+  int64_t r, c;
+  int n;  // elements in the piece (4, or fewer at the end of a row)
+};
+
+__device__ __forceinline__ Piece piece_of(uint64_t t, uint32_t cpr, int64_t N) {
+  uint64_t r, q;
+  if (t <= 0xFFFFFFFFull) {
+    r = (uint32_t)t / cpr;
+    q = (uint32_t)t - (uint32_t)r * cpr;
+  } else {
+    r = t / cpr;
+    q = t - r * cpr;
+  }
+  Piece pc;
+  pc.r = (int64_t)r;
+  pc.c = (int64_t)q * 4;
+  pc.n = N - pc.c < 4 ? (int)(N - pc.c) : 4;
+  return pc;
+}
+
+template <typename T>
+__device__ __forceinline__ void sum_piece(const T *__restrict__ ws, int splits, int64_t MN, int64_t N,
+                                          const Piece &pc, T (&v)[4]) {
+  const int64_t base = pc.r * N + pc.c;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] = T(0);
+  if (pc.n == 4 && (N & 3) == 0) {
+    for (int k = 0; k < splits; ++k) {
+      const uint4 w = __ldcs(reinterpret_cast<const uint4 *>(ws + (int64_t)k * MN + base));
+      T x[4];
+      memcpy(x, &w, sizeof w);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) v[i] += x[i];
+    }
+  } else {
+    for (int k = 0; k < splits; ++k)
+      for (int i = 0; i < pc.n; ++i) v[i] += __ldcs(ws + (int64_t)k * MN + base + i);
   }
 }
 
-// Sum the int32 partials; store as int32, or requantised to int16 / int8.
-__global__ void splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int splits, int64_t M,
-                                         int64_t N, void *__restrict__ C, int64_t ldc, int out_bits,
-                                         int shift) {
+__global__ void __launch_bounds__(kThreads)
+    splitk_reduce_bf16_kernel(const float *__restrict__ ws, int splits, int64_t M, int64_t N,
+                              uint16_t *__restrict__ C, int64_t ldc, uint32_t cpr) {
+  griddep_wait();  // the partials come from the GEMM launched just before
+  const uint64_t t = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (uint64_t)M * cpr) return;
+  const Piece pc = piece_of(t, cpr, N);
+  float v[4];
+  sum_piece(ws, splits, M * N, N, pc, v);
+  uint16_t *dst = C + pc.r * ldc + pc.c;
+  uint16_t h[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const __nv_bfloat16 b = __float2bfloat16_rn(v[i]);  // round once, nearest even
+    h[i] = *reinterpret_cast<const uint16_t *>(&b);
+  }
+  if (pc.n == 4 && (reinterpret_cast<uintptr_t>(dst) & 7) == 0) {
+    *reinterpret_cast<uint2 *>(dst) = make_uint2(h[0] | ((uint32_t)h[1] << 16), h[2] | ((uint32_t)h[3] << 16));
+  } else {
+    for (int i = 0; i < pc.n; ++i) dst[i] = h[i];
+  }
+}
+
+// int32 partials; stored as int32, or requantised to int16 / int8.
+__global__ void __launch_bounds__(kThreads)
+    splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int splits, int64_t M, int64_t N, void *__restrict__ C,
+                             int64_t ldc, int out_bits, int shift, uint32_t cpr) {
   griddep_wait();
-  const int64_t total = M * N;
-  const int32_t hi = out_bits == 32 ? INT32_MAX : (1 << (out_bits - 1)) - 1, lo = -hi - 1;
-  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
-       t += (int64_t)gridDim.x * blockDim.x) {
-    int32_t s = 0;
-    for (int k = 0; k < splits; ++k) s += ws[(int64_t)k * total + t];
-    const int64_t r = t / N, c = t - r * N;
-    if (out_bits == 32)
-      static_cast<int32_t *>(C)[r * ldc + c] = s;
-    else if (out_bits == 16)
-      static_cast<int16_t *>(C)[r * ldc + c] = (int16_t)requantize_s32(s, shift, lo, hi);
+  const uint64_t t = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (uint64_t)M * cpr) return;
+  const Piece pc = piece_of(t, cpr, N);
+  int32_t v[4];
+  sum_piece(ws, splits, M * N, N, pc, v);
+  if (out_bits == 32) {
+    int32_t *dst = static_cast<int32_t *>(C) + pc.r * ldc + pc.c;
+    if (pc.n == 4 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0)
+      *reinterpret_cast<int4 *>(dst) = make_int4(v[0], v[1], v[2], v[3]);
     else
-      static_cast<int8_t *>(C)[r * ldc + c] = (int8_t)requantize_s32(s, shift, lo, hi);
+      for (int i = 0; i < pc.n; ++i) dst[i] = v[i];
+    return;
+  }
+  const int32_t hi = (1 << (out_bits - 1)) - 1, lo = -hi - 1;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] = requantize_s32(v[i], shift, lo, hi);
+  if (out_bits == 16) {
+    int16_t *dst = static_cast<int16_t *>(C) + pc.r * ldc + pc.c;
+    if (pc.n == 4 && (reinterpret_cast<uintptr_t>(dst) & 7) == 0)
+      *reinterpret_cast<uint2 *>(dst) = make_uint2(((uint32_t)v[0] & 0xFFFFu) | ((uint32_t)v[1] << 16),
+                                                   ((uint32_t)v[2] & 0xFFFFu) | ((uint32_t)v[3] << 16));
+    else
+      for (int i = 0; i < pc.n; ++i) dst[i] = (int16_t)v[i];
+  } else {
+    int8_t *dst = static_cast<int8_t *>(C) + pc.r * ldc + pc.c;
+    if (pc.n == 4 && (reinterpret_cast<uintptr_t>(dst) & 3) == 0)
+      *reinterpret_cast<uint32_t *>(dst) = ((uint32_t)v[0] & 0xFFu) | (((uint32_t)v[1] & 0xFFu) << 8) |
+                                           (((uint32_t)v[2] & 0xFFu) << 16) | ((uint32_t)v[3] << 24);
+    else
+      for (int i = 0; i < pc.n; ++i) dst[i] = (int8_t)v[i];
   }
 }
 
@@ -189,14 +292,7 @@ cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStre
 }
 
 cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cudaStream_t st) {
-  static int blocks_per_sm = 0;  // resident blocks per SM (same on every GB300)
-  if (blocks_per_sm == 0) {
-    int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, s8_to_bf16_pair_kernel, kS8Threads, 0) != cudaSuccess ||
-        n < 1)
-      n = 4;
-    blocks_per_sm = n;
-  }
+  (void)sms;  // both kernels cover their work with one thread per piece
   auto dense = [](const S8Job &j) {
     return j.ld_src == j.cols && j.ld_dst == j.cols && (reinterpret_cast<uintptr_t>(j.src) & 15) == 0 &&
            (reinterpret_cast<uintptr_t>(j.dst) & 15) == 0;
@@ -208,19 +304,21 @@ cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cuda
     s8_to_bf16_dense_kernel<<<(unsigned)((vecs + kS8Threads - 1) / kS8Threads), kS8Threads, 0, st>>>(a, b, na, nb);
     return cudaGetLastError();
   }
-  const int64_t cpr_a = (a.cols + kS8Chunk - 1) / kS8Chunk, cpr_b = (b.cols + kS8Chunk - 1) / kS8Chunk;
-  const int64_t items_a = a.rows * cpr_a, items = items_a + b.rows * cpr_b;
+  const uint64_t cpr_a = (uint64_t)(a.cols + 3) / 4, cpr_b = (uint64_t)(b.cols + 3) / 4;
+  const uint64_t items_a = (uint64_t)a.rows * cpr_a, items = items_a + (uint64_t)b.rows * cpr_b;
   if (items == 0) return cudaSuccess;
-  const int64_t want = (items + kS8Threads - 1) / kS8Threads;
-  const int64_t wave = (int64_t)sms * blocks_per_sm;
-  const unsigned grid = (unsigned)(want < wave ? want : wave);
-  s8_to_bf16_pair_kernel<<<grid, kS8Threads, 0, st>>>(a, b, cpr_a, cpr_b, items_a, items);
+  s8_to_bf16_pair_kernel<<<(unsigned)((items + kS8Threads - 1) / kS8Threads), kS8Threads, 0, st>>>(
+      a, b, (uint32_t)(cpr_a ? cpr_a : 1), (uint32_t)(cpr_b ? cpr_b : 1), items_a, items);
   return cudaGetLastError();
 }
 
 cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int64_t ld_src,
                             uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st) {
-  pack_u16_kernel<<<grid_for(rows * cols, 4, sms), kThreads, 0, st>>>(src, rows, cols, ld_src, dst, ld_dst);
+  (void)sms;
+  const uint64_t cpr = (uint64_t)(cols + 3) / 4, items = (uint64_t)rows * cpr;
+  if (items == 0) return cudaSuccess;
+  pack_u16_kernel<<<(unsigned)((items + kS8Threads - 1) / kS8Threads), kS8Threads, 0, st>>>(
+      src, cols, ld_src, dst, ld_dst, (uint32_t)cpr, items);
   return cudaGetLastError();
 }
 
@@ -238,14 +336,18 @@ cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esi
 
 cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, int64_t N,
                                       uint16_t *C, int64_t ldc, int sms, cudaStream_t st) {
-  return launch_ex(splitk_reduce_bf16_kernel, dim3(grid_for(M * N, 2, sms)), dim3(kThreads), 0, st, 1, ws, splits,
-                   M, N, C, ldc);
+  (void)sms;
+  const uint64_t cpr = (uint64_t)(N + 3) / 4, items = (uint64_t)M * cpr;
+  return launch_ex(splitk_reduce_bf16_kernel, dim3((unsigned)((items + kThreads - 1) / kThreads)), dim3(kThreads),
+                   0, st, 1, ws, splits, M, N, C, ldc, (uint32_t)cpr);
 }
 
 cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N, void *C,
                                      int64_t ldc, int out_bits, int shift, int sms, cudaStream_t st) {
-  return launch_ex(splitk_reduce_s32_kernel, dim3(grid_for(M * N, 2, sms)), dim3(kThreads), 0, st, 1, ws, splits,
-                   M, N, C, ldc, out_bits, shift);
+  (void)sms;
+  const uint64_t cpr = (uint64_t)(N + 3) / 4, items = (uint64_t)M * cpr;
+  return launch_ex(splitk_reduce_s32_kernel, dim3((unsigned)((items + kThreads - 1) / kThreads)), dim3(kThreads),
+                   0, st, 1, ws, splits, M, N, C, ldc, out_bits, shift, (uint32_t)cpr);
 }
 
 }  // namespace gb300
