@@ -152,6 +152,20 @@ bool encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2-D (C) or 3-D (split-K partials: N x M x splits) tensor map for the
+// epilogue's TMA stores: boxes of 32 columns x 32 rows (x 1 split).
+bool encode_out(CUtensorMap *map, CUtensorMapDataType type, uint32_t esize, const void *base, uint64_t N,
+                uint64_t M, uint64_t ld, uint64_t splits) {
+  const cuuint64_t dims[3] = {N, M, splits};
+  const cuuint64_t strides[2] = {ld * esize, ld * esize * M};
+  const cuuint32_t box[3] = {32, 32, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUtensorMapSwizzle sw = esize == 4 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+  return g_encode(map, type, splits > 1 ? 3 : 2, const_cast<void *>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 gemm_status_t check_common(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,
                            int64_t ldb, int layout, const void *C, int64_t ldc) {
   if (M < 0 || N < 0 || K < 0) return GEMM_ERR_INVALID_ARG;
@@ -253,7 +267,17 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
   const int64_t kb_per = ceil_div(num_kb, splits);
   splits = ceil_div(num_kb, kb_per);
-  pl.v = TcVariant{bn, b_kmajor, epi, pair};
+  // Output path: the bf16 224-wide kernels keep a pipeline stage instead of
+  // TMA staging blocks; for int8 at 192/224, TMA stores win up to 128 K
+  // steps per unit, beyond which the extra stage wins (measured on GB300: 4096^3 and
+  // 2048 x 11008 x 4096 faster with TMA stores, 2048 x 4096 x 11008 with
+  // the extra stage).
+  bool tma_out;
+  if (epi == kEpiBf16)
+    tma_out = pair ? tc2_bf16_tma_out(bn) : tc_bf16_tma_out(bn);
+  else
+    tma_out = (bn != 224 && bn != 192) || kb_per <= 128;
+  pl.v = TcVariant{bn, b_kmajor, epi, pair, tma_out};
   TcParams &p = pl.p;
   p.M = (int)M;
   p.N = (int)N;
@@ -273,10 +297,10 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   static const bool debug = env_int("GB300_GEMM_DEBUG") != 0;
   if (debug)
     std::fprintf(stderr,
-                 "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d tiles=%lldx%lld splits=%lld grid=%d "
+                 "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d%s tiles=%lldx%lld splits=%lld grid=%d "
                  "(SMs %d, co-resident pairs %d)\n",
                  (long long)M, (long long)N, (long long)K, epi == kEpiS32 ? "int8" : "bf16",
-                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn, (long long)tiles_m, (long long)tiles_n,
+                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn, tma_out ? " tma-store" : "", (long long)tiles_m, (long long)tiles_n,
                  (long long)splits, pl.grid, sms, pairs);
   return pl;
 }
@@ -303,17 +327,40 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   p.ldc = ldc;
   p.c_vec = aligned16(C) && ((ldc * esize) % 16 == 0);
   p.ws = partials;
+  // Epilogue stores through TMA where the output allows it: bf16 or int32
+  // C with a 16-byte aligned base and pitch; split-K partials when their
+  // pitch (N words) is a multiple of 16 bytes.  int16 / int8 outputs and
+  // other cases store directly (GB300_GEMM_TMA_STORE=0 forces that).
+  CUtensorMap tout = tb;
+  p.out_tma = kOutDirect;
+  const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
+  if (pl.v.tma_out && !(tma_env && std::atoi(tma_env) == 0)) {
+    const bool s32 = pl.v.epi == kEpiS32;
+    if (p.splits > 1) {
+      if (p.N % 4 == 0) {
+        if (!encode_out(&tout, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, partials,
+                        (uint64_t)p.N, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.splits))
+          return GEMM_ERR_CUDA;
+        p.out_tma = kOutTmaWs;
+      }
+    } else if ((!s32 || p.out_bits == 32) && p.c_vec) {
+      if (!encode_out(&tout, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, s32 ? 4 : 2,
+                      C, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ldc, 1))
+        return GEMM_ERR_CUDA;
+      p.out_tma = kOutTmaC;
+    }
+  }
   p.err = d.err;
   p.wait_limit_ns = wait_limit_ns();
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
   cudaError_t e;
   if (pl.v.pair)
-    e = pl.v.epi == kEpiS32 ? launch_tc2_s32(pl.v, ta, tb, p, pl.grid, st)
-                            : launch_tc2_bf16(pl.v, ta, tb, p, pl.grid, st);
+    e = pl.v.epi == kEpiS32 ? launch_tc2_s32(pl.v, ta, tb, tout, p, pl.grid, st)
+                            : launch_tc2_bf16(pl.v, ta, tb, tout, p, pl.grid, st);
   else
-    e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, p, pl.grid, st)
-                            : launch_tc_bf16(pl.v, ta, tb, p, pl.grid, st);
+    e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, tout, p, pl.grid, st)
+                            : launch_tc_bf16(pl.v, ta, tb, tout, p, pl.grid, st);
   g_launches.fetch_add(1);
   if (e != cudaSuccess) return GEMM_ERR_CUDA;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;

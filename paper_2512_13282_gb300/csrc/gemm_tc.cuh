@@ -15,7 +15,14 @@
 //                      tile overwrites instead of accumulating, which takes
 //                      the place of the paper's zeroing kernel (Sec. 4.2.1).
 //   warps 2..          epilogue: TMEM -> registers -> bf16 (RNE) or int32 ->
-//                      global memory, masked at the M/N edges.  Two
+//                      a 32-row x 32-column block in the warp's own shared
+//                      memory (swizzled as the TMA expects) -> one TMA tensor
+//                      store per block, which writes whole lines of C and
+//                      clips at the M/N edges (stores that each lane makes to
+//                      its own row would touch 32 lines per instruction and
+//                      compete with the operand traffic; where C's address
+//                      or pitch rules TMA out, or for int16/int8 outputs,
+//                      lanes store their rows directly).  Two
 //                      accumulators let the epilogue of one tile overlap the
 //                      main loop of the next (the paper keeps a single C
 //                      buffer for lack of L1 space, Sec. 5.3.2; TMEM has room
@@ -62,7 +69,11 @@ struct TcParams {
   uint64_t wait_limit_ns;
   int out_bits;      // int8 path: 32 (exact int32 C), 16 or 8 (requantised C)
   int out_shift;     // int8 path with out_bits < 32: right shift, 0..31
+  int out_tma;       // kOutDirect, kOutTmaC (tmOut maps C) or kOutTmaWs (tmOut maps the partials)
 };
+
+// How the epilogue writes its results.
+enum OutMode : int { kOutDirect = 0, kOutTmaC = 1, kOutTmaWs = 2 };
 
 __host__ __device__ constexpr uint32_t pow2_at_least(uint32_t x) {
   uint32_t p = 32;
@@ -70,7 +81,7 @@ __host__ __device__ constexpr uint32_t pow2_at_least(uint32_t x) {
   return p;
 }
 
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
 struct TcCfg {
   // MMA N for M = 128 is a multiple of 16 up to 256; the epilogue moves 32
   // columns per TMEM load; an MN-major B tile is assembled from 64-wide boxes.
@@ -83,7 +94,11 @@ struct TcCfg {
   static constexpr int kThreads = (2 + EPI_WARPS) * 32;
   static constexpr int kColsPerThread = BN / (EPI_WARPS / 4);
   static_assert(kColsPerThread % 16 == 0, "epilogue chunks are 32 columns, plus one of 16");
-  static constexpr uint32_t kBarOffset = STAGES * kStageBytes;
+  // TMA_OUT: per epilogue warp, one 32 x 32 block of 32-bit words (int32
+  // results or split-K partials of either path; bf16 results use half of it)
+  static constexpr uint32_t kEpiWarpBytes = TMA_OUT ? 4096 : 0;
+  static constexpr uint32_t kEpiOffset = STAGES * kStageBytes;  // 1024-byte aligned
+  static constexpr uint32_t kBarOffset = kEpiOffset + EPI_WARPS * kEpiWarpBytes;
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
@@ -231,6 +246,53 @@ __device__ __forceinline__ void store_s8_result(const TcParams &p, int64_t row, 
   }
 }
 
+// TMA-store epilogue.  A warp stages 32 rows (lane = row) x 32 columns in
+// its shared-memory block laid out as the tensor map's swizzle expects, then
+// lane 0 stores the block with one TMA tensor store.  The block is reused
+// once the previous store has read it.  `in_range`: the block's first row
+// and column lie inside the output (the TMA clips the rest).
+//
+// 32-bit words (int32 results, fp32/int32 split-K partials): 128-byte rows,
+// 128-byte swizzle (16-byte chunk j of row r lands at chunk j ^ (r % 8)).
+template <bool WS>
+__device__ __forceinline__ void tma_out_words32(const CUtensorMap *tm, uint32_t buf, int lane,
+                                                const uint32_t (&v)[32], int x, int y, int z, bool in_range) {
+  if (lane == 0) bulk_wait_read_all();
+  __syncwarp();
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    st_shared_v4(buf + lane * 128 + ((j ^ (lane & 7)) << 4), v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0 && in_range) {
+    if constexpr (WS)
+      tma_store_3d(tm, buf, x, y, z);
+    else
+      tma_store_2d(tm, buf, x, y);
+    bulk_commit();
+  }
+}
+
+// bf16 results: 32 fp32 accumulator words rounded to 32 bf16 (64-byte rows),
+// 64-byte swizzle (chunk j of row r lands at chunk j ^ ((r / 2) % 4)).
+__device__ __forceinline__ void tma_out_bf16x32(const CUtensorMap *tm, uint32_t buf, int lane, const uint32_t (&r)[32],
+                                                int x, int y, bool in_range) {
+  uint32_t h[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) h[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+  if (lane == 0) bulk_wait_read_all();
+  __syncwarp();
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    st_shared_v4(buf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4), h[4 * j], h[4 * j + 1], h[4 * j + 2], h[4 * j + 3]);
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0 && in_range) {
+    tma_store_2d(tm, buf, x, y);
+    bulk_commit();
+  }
+}
+
 template <int W>
 __device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
   if constexpr (W == 32)
@@ -239,11 +301,12 @@ __device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
     tmem_ld_32x32b_x16(taddr, r);
 }
 
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
-__global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::kThreads, 1)
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
+__global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const TcParams p) {
-  using Cfg = TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>;
+                   const __grid_constant__ CUtensorMap tmOut, const TcParams p) {
+  using Cfg = TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>;
+  const int out_tma = TMA_OUT ? p.out_tma : (int)kOutDirect;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-byte alignment
@@ -277,6 +340,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    if (out_tma != kOutDirect) tma_prefetch_desc(&tmOut);
   }
   if (warp == 1) tmem_alloc<Cfg::kTmemCols>(smem_addr(tmem_slot));
   tc_fence_before_sync();
@@ -381,6 +445,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
     const int row_in_tile = quad * 32 + lane;
     const bool split = p.splits > 1;
     const bool ws_vec = (p.N & 3) == 0;
+    const uint32_t ebuf = base + Cfg::kEpiOffset + ew * Cfg::kEpiWarpBytes;
     uint32_t acc_cnt = 0;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
@@ -388,6 +453,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
       const int64_t row = (int64_t)w.tm * kBM + row_in_tile;
       const bool row_ok = row < p.M;
       const int col0 = w.tn * BN + colpart * CPT;
+      const int y0 = w.tm * kBM + quad * 32;  // first row of this warp's blocks
       if constexpr (EPI == kEpiS32) {
         int32_t acc[CPT];
 #pragma unroll
@@ -422,10 +488,34 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
           ++acc_cnt;
         }
         if (!ok) break;
-        if (row_ok) {
-          // split-K partials stay int32; the reduction requantises
-          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
-                                 : nullptr;
+        // split-K partials stay int32; the reduction requantises
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                               : nullptr;
+        if (out_tma != kOutDirect) {
+#pragma unroll
+          for (int c = 0; c < CPT / 32; ++c) {
+            uint32_t v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
+            const int x = col0 + c * 32;
+            if (out_tma == kOutTmaWs)
+              tma_out_words32<true>(&tmOut, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
+            else
+              tma_out_words32<false>(&tmOut, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+          }
+          if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
+            constexpr int kTail = (CPT / 32) * 32;
+            if (row_ok) {
+              uint32_t v[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
+              if (split)
+                store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+              else
+                store_s8_result<16>(p, row, col0 + kTail, v);
+            }
+          }
+        } else if (row_ok) {
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t v[32];
@@ -455,7 +545,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::k
         }
         tc_fence_after_sync();
         const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
-uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
+        uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
         uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
                                : nullptr;
 #pragma unroll 1
@@ -463,11 +553,17 @@ uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
           uint32_t r[32];
           tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
-          if (!row_ok) continue;
-          if (split)
-            store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, r);
-          else
-            store_bf16<32>(crow, col0 + c * 32, p.N, p.c_vec != 0, r);
+          const int x = col0 + c * 32;
+          if (out_tma == kOutTmaWs) {
+            tma_out_words32<true>(&tmOut, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
+          } else if (out_tma == kOutTmaC) {
+            tma_out_bf16x32(&tmOut, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
+          } else if (row_ok) {
+            if (split)
+              store_words<32>(wrow, x, p.N, ws_vec, r);
+            else
+              store_bf16<32>(crow, x, p.N, p.c_vec != 0, r);
+          }
         }
         if constexpr (CPT % 32 != 0) {
           constexpr int kTail = (CPT / 32) * 32;
@@ -488,6 +584,7 @@ uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
     }
   }
 
+  if (TMA_OUT && warp >= 2 && lane == 0) bulk_wait_all();  // this warp's TMA stores have landed
   griddep_launch_dependents();  // e.g. the split-K reduction may start setting up
   __syncwarp();
   tc_fence_before_sync();

@@ -90,7 +90,7 @@ __device__ __forceinline__ void tc_commit_pair_multicast(uint32_t bar) {
       : "memory");
 }
 
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
 struct Tc2Cfg {
   static constexpr int kHalfN = BN / 2;  // B extent (in N) each CTA loads
   static_assert(kHalfN % 16 == 0 && BN <= 256, "pair MMA N is a multiple of 32 up to 256");
@@ -103,7 +103,9 @@ struct Tc2Cfg {
   static constexpr int kEpiThreads = EPI_WARPS * 32;
   static constexpr int kColsPerThread = BN / (EPI_WARPS / 4);
   static_assert(kColsPerThread % 16 == 0, "epilogue chunks are 32 columns, plus one of 16");
-  static constexpr uint32_t kBarOffset = STAGES * kStageBytes;
+  static constexpr uint32_t kEpiWarpBytes = TMA_OUT ? 4096 : 0;  // one 32 x 32 block of 32-bit words
+  static constexpr uint32_t kEpiOffset = STAGES * kStageBytes;
+  static constexpr uint32_t kBarOffset = kEpiOffset + EPI_WARPS * kEpiWarpBytes;
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
@@ -112,11 +114,12 @@ struct Tc2Cfg {
 
 // Launch with cluster dimensions (2,1,1) and an even grid; tiles_m counts
 // 256-row tiles.
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS>
-__global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::kThreads, 1)
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
+__global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>::kThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const TcParams p) {
-  using Cfg = Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>;
+                    const __grid_constant__ CUtensorMap tmOut, const TcParams p) {
+  using Cfg = Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>;
+  const int out_tma = TMA_OUT ? p.out_tma : (int)kOutDirect;
   constexpr int kTileM = 2 * kBM;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -155,6 +158,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
     fence_mbar_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    if (out_tma != kOutDirect) tma_prefetch_desc(&tmOut);
   }
   __syncwarp();
   if (warp == 1) tmem_alloc_pair<Cfg::kTmemCols>(smem_addr(tmem_slot));
@@ -265,6 +269,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
     const int row_in_tile = (int)rank * kBM + quad * 32 + lane;
     const bool split = p.splits > 1;
     const bool ws_vec = (p.N & 3) == 0;
+    const uint32_t ebuf = base + Cfg::kEpiOffset + ew * Cfg::kEpiWarpBytes;
     uint32_t acc_cnt = 0;
     bool ok = true;
     for (int u = cluster; ok && u < num_units; u += num_clusters) {
@@ -272,6 +277,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
       const int64_t row = (int64_t)w.tm * kTileM + row_in_tile;
       const bool row_ok = row < p.M;
       const int col0 = w.tn * BN + colpart * CPT;
+      const int y0 = w.tm * kTileM + (int)rank * kBM + quad * 32;  // first row of this warp's blocks
       if constexpr (EPI == kEpiS32) {
         int32_t acc[CPT];
 #pragma unroll
@@ -305,10 +311,34 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
           ++acc_cnt;
         }
         if (!ok) break;
-        if (row_ok) {
-          // split-K partials stay int32; the reduction requantises
-          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
-                                 : nullptr;
+        // split-K partials stay int32; the reduction requantises
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                               : nullptr;
+        if (out_tma != kOutDirect) {
+#pragma unroll
+          for (int c = 0; c < CPT / 32; ++c) {
+            uint32_t v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
+            const int x = col0 + c * 32;
+            if (out_tma == kOutTmaWs)
+              tma_out_words32<true>(&tmOut, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
+            else
+              tma_out_words32<false>(&tmOut, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+          }
+          if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
+            constexpr int kTail = (CPT / 32) * 32;
+            if (row_ok) {
+              uint32_t v[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
+              if (split)
+                store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+              else
+                store_s8_result<16>(p, row, col0 + kTail, v);
+            }
+          }
+        } else if (row_ok) {
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t v[32];
@@ -346,11 +376,17 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
           uint32_t r[32];
           tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
-          if (!row_ok) continue;
-          if (split)
-            store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, r);
-          else
-            store_bf16<32>(crow, col0 + c * 32, p.N, p.c_vec != 0, r);
+          const int x = col0 + c * 32;
+          if (out_tma == kOutTmaWs) {
+            tma_out_words32<true>(&tmOut, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
+          } else if (out_tma == kOutTmaC) {
+            tma_out_bf16x32(&tmOut, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
+          } else if (row_ok) {
+            if (split)
+              store_words<32>(wrow, x, p.N, ws_vec, r);
+            else
+              store_bf16<32>(crow, x, p.N, p.c_vec != 0, r);
+          }
         }
         if constexpr (CPT % 32 != 0) {
           constexpr int kTail = (CPT / 32) * 32;
@@ -371,6 +407,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS>::
     }
   }
 
+  if (TMA_OUT && warp >= 2 && lane == 0) bulk_wait_all();  // this warp's TMA stores have landed
   griddep_launch_dependents();  // e.g. the split-K reduction may start setting up
   __syncwarp();
   tc_fence_before_sync();

@@ -6,11 +6,12 @@
 
 namespace gb300 {
 
-template <int BN, int STAGES, bool KM, int EPI, int EW>
-cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const TcParams &p, int grid,
+template <int BN, int STAGES, bool KM, int EPI, int EW, bool TMA>
+cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
+                        int grid,
                         cudaStream_t st) {
-  using Cfg = Tc2Cfg<BN, STAGES, KM, EPI, EW>;
-  auto kern = gemm_tc2_kernel<BN, STAGES, KM, EPI, EW>;
+  using Cfg = Tc2Cfg<BN, STAGES, KM, EPI, EW, TMA>;
+  auto kern = gemm_tc2_kernel<BN, STAGES, KM, EPI, EW, TMA>;
   static bool opted_in[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -21,7 +22,7 @@ cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const TcPara
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
   // grid is even: a whole number of pairs
-  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 2, a, b, p);
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 2, a, b, o, p);
 }
 
 }  // namespace gb300

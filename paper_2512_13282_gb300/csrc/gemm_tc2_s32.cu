@@ -1,22 +1,27 @@
 // Instantiations of the CTA-pair tcgen05 kernel with the exact int32 (slab)
-// epilogue.
+// epilogue: TMA stores through eight 4 KB staging blocks (6 stages for
+// 192-256, 8 for 128); 192 and 224 also come with 7 stages and direct
+// stores for long reductions (the planner's choice, v.tma_out).
 #include "gemm_tc2_launch.cuh"
 
 namespace gb300 {
 
 cudaError_t launch_tc2_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                           const TcParams &p, int grid, cudaStream_t st) {
+                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
+  const bool t = v.tma_out;
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_pair<256, 6, true, kEpiS32, 8>(a, b, p, grid, st);
-      case 224: return launch_pair<224, 7, true, kEpiS32, 8>(a, b, p, grid, st);
-      case 192: return launch_pair<192, 7, true, kEpiS32, 8>(a, b, p, grid, st);
-      case 128: return launch_pair<128, 8, true, kEpiS32, 4>(a, b, p, grid, st);
+      case 256: return launch_pair<256, 6, true, kEpiS32, 8, true>(a, b, o, p, grid, st);
+      case 224: return t ? launch_pair<224, 6, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
+                         : launch_pair<224, 7, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
+      case 192: return t ? launch_pair<192, 6, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
+                         : launch_pair<192, 7, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
+      case 128: return launch_pair<128, 8, true, kEpiS32, 4, true>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_pair<256, 6, false, kEpiS32, 8>(a, b, p, grid, st);
-      case 128: return launch_pair<128, 8, false, kEpiS32, 4>(a, b, p, grid, st);
+      case 256: return launch_pair<256, 6, false, kEpiS32, 8, true>(a, b, o, p, grid, st);
+      case 128: return launch_pair<128, 8, false, kEpiS32, 4, true>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;

@@ -4,11 +4,12 @@
 namespace gb300 {
 
 namespace {
-template <int BN, int STAGES, bool KM, int EPI, int EW>
-cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParams &p, int grid,
+template <int BN, int STAGES, bool KM, int EPI, int EW, bool TMA>
+cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
+                       int grid,
                        cudaStream_t st) {
-  using Cfg = TcCfg<BN, STAGES, KM, EPI, EW>;
-  auto kern = gemm_tc_kernel<BN, STAGES, KM, EPI, EW>;
+  using Cfg = TcCfg<BN, STAGES, KM, EPI, EW, TMA>;
+  auto kern = gemm_tc_kernel<BN, STAGES, KM, EPI, EW, TMA>;
   // the shared-memory opt-in is per device and kernel: set it once
   static bool opted_in[64] = {};
   int dev = 0;
@@ -19,29 +20,34 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParam
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
-  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, p);
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, o, p);
 }
 }  // namespace
 
-// Tile widths compiled for the bf16 epilogue: 128 (6 stages), 192 (5),
-// 224 (5, B column-major only), 256 (4).
+// Tile widths compiled for the bf16 epilogue, with their stage counts and
+// output path (TMA stores through four 4 KB staging blocks, or direct
+// stores where the staging blocks would cost a pipeline stage): 128 (6,
+// TMA), 192 (5, TMA), 224 (5, direct; B column-major only), 256 (4, TMA).
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                           const TcParams &p, int grid, cudaStream_t st) {
+                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_one<256, 4, true, kEpiBf16, 4>(a, b, p, grid, st);
-      case 224: return launch_one<224, 5, true, kEpiBf16, 4>(a, b, p, grid, st);
-      case 192: return launch_one<192, 5, true, kEpiBf16, 4>(a, b, p, grid, st);
-      case 128: return launch_one<128, 6, true, kEpiBf16, 4>(a, b, p, grid, st);
+      case 256: return launch_one<256, 4, true, kEpiBf16, 4, true>(a, b, o, p, grid, st);
+      case 224: return launch_one<224, 5, true, kEpiBf16, 4, false>(a, b, o, p, grid, st);
+      case 192: return launch_one<192, 5, true, kEpiBf16, 4, true>(a, b, o, p, grid, st);
+      case 128: return launch_one<128, 6, true, kEpiBf16, 4, true>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_one<256, 4, false, kEpiBf16, 4>(a, b, p, grid, st);
-      case 192: return launch_one<192, 5, false, kEpiBf16, 4>(a, b, p, grid, st);
-      case 128: return launch_one<128, 6, false, kEpiBf16, 4>(a, b, p, grid, st);
+      case 256: return launch_one<256, 4, false, kEpiBf16, 4, true>(a, b, o, p, grid, st);
+      case 192: return launch_one<192, 5, false, kEpiBf16, 4, true>(a, b, o, p, grid, st);
+      case 128: return launch_one<128, 6, false, kEpiBf16, 4, true>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;
 }
+
+// Whether launch_tc_bf16's variant for this tile width stores through TMA.
+bool tc_bf16_tma_out(int bn) { return bn != 224; }
 
 }  // namespace gb300

@@ -4,11 +4,12 @@
 namespace gb300 {
 
 namespace {
-template <int BN, int STAGES, bool KM, int EPI, int EW>
-cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParams &p, int grid,
+template <int BN, int STAGES, bool KM, int EPI, int EW, bool TMA>
+cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
+                       int grid,
                        cudaStream_t st) {
-  using Cfg = TcCfg<BN, STAGES, KM, EPI, EW>;
-  auto kern = gemm_tc_kernel<BN, STAGES, KM, EPI, EW>;
+  using Cfg = TcCfg<BN, STAGES, KM, EPI, EW, TMA>;
+  auto kern = gemm_tc_kernel<BN, STAGES, KM, EPI, EW, TMA>;
   // the shared-memory opt-in is per device and kernel: set it once
   static bool opted_in[64] = {};
   int dev = 0;
@@ -19,24 +20,34 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const TcParam
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
-  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, p);
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, o, p);
 }
 }  // namespace
 
 // Tile widths compiled for the int32 epilogue: 128 (one epilogue warpgroup,
-// 128 int32 accumulators per thread), 192, 224 (B column-major only) and 256
-// (two warpgroups, 96 / 112 / 128 per thread).
+// 128 int32 accumulators per thread, 6 stages), 192, 224 (B column-major
+// only) and 256 (two warpgroups, 96 / 112 / 128 per thread).  With TMA
+// stores, eight 4 KB staging blocks sit beside the ring (4 stages for
+// 192-256); 192 and 224 also come with 5 stages and direct stores, which
+// long reductions prefer (the planner's choice, v.tma_out).
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                          const TcParams &p, int grid, cudaStream_t st) {
+                          const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
+  const bool km = v.b_kmajor, t = v.tma_out;
   switch (v.bn) {
-    case 256: return v.b_kmajor ? launch_one<256, 4, true, kEpiS32, 8>(a, b, p, grid, st)
-                                : launch_one<256, 4, false, kEpiS32, 8>(a, b, p, grid, st);
-    case 224: return v.b_kmajor ? launch_one<224, 5, true, kEpiS32, 8>(a, b, p, grid, st)
-                                : cudaErrorInvalidValue;
-    case 192: return v.b_kmajor ? launch_one<192, 5, true, kEpiS32, 8>(a, b, p, grid, st)
-                                : launch_one<192, 5, false, kEpiS32, 8>(a, b, p, grid, st);
-    case 128: return v.b_kmajor ? launch_one<128, 6, true, kEpiS32, 4>(a, b, p, grid, st)
-                                : launch_one<128, 6, false, kEpiS32, 4>(a, b, p, grid, st);
+    case 256: return km ? launch_one<256, 4, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
+                        : launch_one<256, 4, false, kEpiS32, 8, true>(a, b, o, p, grid, st);
+    case 224:
+      if (!km) return cudaErrorInvalidValue;
+      return t ? launch_one<224, 4, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
+               : launch_one<224, 5, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
+    case 192:
+      if (km)
+        return t ? launch_one<192, 4, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
+                 : launch_one<192, 5, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
+      return t ? launch_one<192, 4, false, kEpiS32, 8, true>(a, b, o, p, grid, st)
+               : launch_one<192, 5, false, kEpiS32, 8, false>(a, b, o, p, grid, st);
+    case 128: return km ? launch_one<128, 6, true, kEpiS32, 4, true>(a, b, o, p, grid, st)
+                        : launch_one<128, 6, false, kEpiS32, 4, true>(a, b, o, p, grid, st);
   }
   return cudaErrorInvalidValue;
 }
