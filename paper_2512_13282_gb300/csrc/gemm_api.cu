@@ -160,7 +160,10 @@ bool encode_out(CUtensorMap *map, CUtensorMapDataType type, uint32_t esize, cons
   const cuuint64_t strides[2] = {ld * esize, ld * esize * M};
   const cuuint32_t box[3] = {32, 32, 1};
   const cuuint32_t estr[3] = {1, 1, 1};
-  const CUtensorMapSwizzle sw = esize == 4 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+  // 32 columns per box: 128-, 64- or 32-byte rows, swizzled to match
+  const CUtensorMapSwizzle sw = esize == 4   ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : esize == 2 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                             : CU_TENSOR_MAP_SWIZZLE_32B;
   return g_encode(map, type, splits > 1 ? 3 : 2, const_cast<void *>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -331,11 +334,15 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   // C with a 16-byte aligned base and pitch; split-K partials when their
   // pitch (N words) is a multiple of 16 bytes.  int16 / int8 outputs and
   // other cases store directly (GB300_GEMM_TMA_STORE=0 forces that).
+  const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
+  const bool s32 = pl.v.epi == kEpiS32;
+  const bool tma_ok = !(tma_env && std::atoi(tma_env) == 0) && (p.splits > 1 ? p.N % 4 == 0 : p.c_vec != 0);
+  // An output that will be stored directly wants the variant with the extra
+  // pipeline stage where one exists (int8 at 192 / 224).
+  if (!tma_ok && s32 && (pl.v.bn == 192 || pl.v.bn == 224)) pl.v.tma_out = false;
   CUtensorMap tout = tb;
   p.out_tma = kOutDirect;
-  const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
-  if (pl.v.tma_out && !(tma_env && std::atoi(tma_env) == 0)) {
-    const bool s32 = pl.v.epi == kEpiS32;
+  if (pl.v.tma_out && tma_ok) {
     if (p.splits > 1) {
       if (p.N % 4 == 0) {
         if (!encode_out(&tout, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, partials,
@@ -343,9 +350,12 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
           return GEMM_ERR_CUDA;
         p.out_tma = kOutTmaWs;
       }
-    } else if ((!s32 || p.out_bits == 32) && p.c_vec) {
-      if (!encode_out(&tout, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, s32 ? 4 : 2,
-                      C, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ldc, 1))
+    } else if (p.c_vec) {
+      const CUtensorMapDataType type = !s32                ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16
+                                       : p.out_bits == 32 ? CU_TENSOR_MAP_DATA_TYPE_INT32
+                                       : p.out_bits == 16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16
+                                                          : CU_TENSOR_MAP_DATA_TYPE_UINT8;
+      if (!encode_out(&tout, type, (uint32_t)esize, C, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ldc, 1))
         return GEMM_ERR_CUDA;
       p.out_tma = kOutTmaC;
     }

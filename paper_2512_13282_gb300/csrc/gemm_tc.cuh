@@ -21,8 +21,8 @@
 //                      clips at the M/N edges (stores that each lane makes to
 //                      its own row would touch 32 lines per instruction and
 //                      compete with the operand traffic; where C's address
-//                      or pitch rules TMA out, or for int16/int8 outputs,
-//                      lanes store their rows directly).  Two
+//                      or pitch rules TMA out, lanes store their rows
+//                      directly).  Two
 //                      accumulators let the epilogue of one tile overlap the
 //                      main loop of the next (the paper keeps a single C
 //                      buffer for lack of L1 space, Sec. 5.3.2; TMEM has room
@@ -293,6 +293,48 @@ __device__ __forceinline__ void tma_out_bf16x32(const CUtensorMap *tm, uint32_t 
   }
 }
 
+// Requantised int8-path results (int16 or int8 C): 32 int32 sums of a row
+// requantised and packed into 64-byte (int16; 64-byte swizzle) or 32-byte
+// (int8; 32-byte swizzle: chunk j of row r lands at chunk j ^ ((r / 4) % 2))
+// rows, then stored like the other blocks.
+__device__ __forceinline__ void tma_out_narrow(const CUtensorMap *tm, uint32_t buf, int lane, const uint32_t (&v)[32],
+                                               int bits, int shift, int x, int y, bool in_range) {
+  const int32_t hi = (1 << (bits - 1)) - 1, lo = -hi - 1;
+  uint32_t h[16];
+  if (bits == 16) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      h[i] = ((uint32_t)requantize_s32((int32_t)v[2 * i], shift, lo, hi) & 0xFFFFu) |
+             ((uint32_t)requantize_s32((int32_t)v[2 * i + 1], shift, lo, hi) << 16);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      h[i] = ((uint32_t)requantize_s32((int32_t)v[4 * i], shift, lo, hi) & 0xFFu) |
+             (((uint32_t)requantize_s32((int32_t)v[4 * i + 1], shift, lo, hi) & 0xFFu) << 8) |
+             (((uint32_t)requantize_s32((int32_t)v[4 * i + 2], shift, lo, hi) & 0xFFu) << 16) |
+             ((uint32_t)requantize_s32((int32_t)v[4 * i + 3], shift, lo, hi) << 24);
+  }
+  if (lane == 0) bulk_wait_read_all();
+  __syncwarp();
+  if (bits == 16) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      st_shared_v4(buf + lane * 64 + ((j ^ ((lane >> 1) & 3)) << 4), h[4 * j], h[4 * j + 1], h[4 * j + 2],
+                   h[4 * j + 3]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+      st_shared_v4(buf + lane * 32 + ((j ^ ((lane >> 2) & 1)) << 4), h[4 * j], h[4 * j + 1], h[4 * j + 2],
+                   h[4 * j + 3]);
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0 && in_range) {
+    tma_store_2d(tm, buf, x, y);
+    bulk_commit();
+  }
+}
+
 template <int W>
 __device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
   if constexpr (W == 32)
@@ -500,8 +542,10 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
             const int x = col0 + c * 32;
             if (out_tma == kOutTmaWs)
               tma_out_words32<true>(&tmOut, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
-            else
+            else if (p.out_bits == 32)
               tma_out_words32<false>(&tmOut, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+            else
+              tma_out_narrow(&tmOut, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
           }
           if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
             constexpr int kTail = (CPT / 32) * 32;

@@ -323,8 +323,10 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
             const int x = col0 + c * 32;
             if (out_tma == kOutTmaWs)
               tma_out_words32<true>(&tmOut, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
-            else
+            else if (p.out_bits == 32)
               tma_out_words32<false>(&tmOut, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+            else
+              tma_out_narrow(&tmOut, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
           }
           if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
             constexpr int kTail = (CPT / 32) * 32;
