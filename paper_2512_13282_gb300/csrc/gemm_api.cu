@@ -153,17 +153,18 @@ bool encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t
 }
 
 // 2-D (C) or 3-D (split-K partials: N x M x splits) tensor map for the
-// epilogue's TMA stores: boxes of 32 columns x 32 rows (x 1 split).
+// epilogue's TMA stores: boxes of box_cols columns x 32 rows (x 1 split).
 bool encode_out(CUtensorMap *map, CUtensorMapDataType type, uint32_t esize, const void *base, uint64_t N,
-                uint64_t M, uint64_t ld, uint64_t splits) {
+                uint64_t M, uint64_t ld, uint64_t splits, uint32_t box_cols = 32) {
   const cuuint64_t dims[3] = {N, M, splits};
   const cuuint64_t strides[2] = {ld * esize, ld * esize * M};
-  const cuuint32_t box[3] = {32, 32, 1};
+  const cuuint32_t box[3] = {box_cols, 32, 1};
   const cuuint32_t estr[3] = {1, 1, 1};
-  // 32 columns per box: 128-, 64- or 32-byte rows, swizzled to match
-  const CUtensorMapSwizzle sw = esize == 4   ? CU_TENSOR_MAP_SWIZZLE_128B
-                                : esize == 2 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                             : CU_TENSOR_MAP_SWIZZLE_32B;
+  // 128-, 64- or 32-byte box rows, swizzled to match the staging blocks
+  const uint32_t row_bytes = box_cols * esize;
+  const CUtensorMapSwizzle sw = row_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : row_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                  : CU_TENSOR_MAP_SWIZZLE_32B;
   return g_encode(map, type, splits > 1 ? 3 : 2, const_cast<void *>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -270,16 +271,17 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
   const int64_t kb_per = ceil_div(num_kb, splits);
   splits = ceil_div(num_kb, kb_per);
-  // Output path: the bf16 224-wide kernels keep a pipeline stage instead of
-  // TMA staging blocks; for int8 at 192/224, TMA stores win up to 128 K
-  // steps per unit, beyond which the extra stage wins (measured on GB300: 4096^3 and
-  // 2048 x 11008 x 4096 faster with TMA stores, 2048 x 4096 x 11008 with
+  // Output path: the bf16 224-wide kernels keep a pipeline stage and stage
+  // their TMA stores through 1 KB blocks; for int8 at 192/224, TMA stores
+  // (4 KB blocks, one stage less) win up to 128 K steps per unit, beyond
+  // which the extra stage and direct stores win (measured on GB300: 4096^3
+  // and 2048 x 11008 x 4096 faster with TMA stores, 2048 x 4096 x 11008 with
   // the extra stage).
-  bool tma_out;
+  int tma_out;
   if (epi == kEpiBf16)
     tma_out = pair ? tc2_bf16_tma_out(bn) : tc_bf16_tma_out(bn);
   else
-    tma_out = (bn != 224 && bn != 192) || kb_per <= 128;
+    tma_out = ((bn != 224 && bn != 192) || kb_per <= 128) ? 1 : 0;
   pl.v = TcVariant{bn, b_kmajor, epi, pair, tma_out};
   TcParams &p = pl.p;
   p.M = (int)M;
@@ -303,7 +305,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
                  "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d%s tiles=%lldx%lld splits=%lld grid=%d "
                  "(SMs %d, co-resident pairs %d)\n",
                  (long long)M, (long long)N, (long long)K, epi == kEpiS32 ? "int8" : "bf16",
-                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn, tma_out ? " tma-store" : "", (long long)tiles_m, (long long)tiles_n,
+                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn, tma_out == 2 ? " tma-store-1k" : tma_out ? " tma-store" : "", (long long)tiles_m, (long long)tiles_n,
                  (long long)splits, pl.grid, sms, pairs);
   return pl;
 }
@@ -336,13 +338,14 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   // other cases store directly (GB300_GEMM_TMA_STORE=0 forces that).
   const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
   const bool s32 = pl.v.epi == kEpiS32;
-  const bool tma_ok = !(tma_env && std::atoi(tma_env) == 0) && (p.splits > 1 ? p.N % 4 == 0 : p.c_vec != 0);
+  const bool tma_ok = !(tma_env && std::atoi(tma_env) == 0) &&
+                      (p.splits > 1 ? p.N % 4 == 0 && pl.v.tma_out == 1 : p.c_vec != 0);
   // An output that will be stored directly wants the variant with the extra
   // pipeline stage where one exists (int8 at 192 / 224).
-  if (!tma_ok && s32 && (pl.v.bn == 192 || pl.v.bn == 224)) pl.v.tma_out = false;
+  if (!tma_ok && s32 && (pl.v.bn == 192 || pl.v.bn == 224)) pl.v.tma_out = 0;
   CUtensorMap tout = tb;
   p.out_tma = kOutDirect;
-  if (pl.v.tma_out && tma_ok) {
+  if (pl.v.tma_out != 0 && tma_ok) {
     if (p.splits > 1) {
       if (p.N % 4 == 0) {
         if (!encode_out(&tout, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, partials,
@@ -355,7 +358,8 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
                                        : p.out_bits == 32 ? CU_TENSOR_MAP_DATA_TYPE_INT32
                                        : p.out_bits == 16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16
                                                           : CU_TENSOR_MAP_DATA_TYPE_UINT8;
-      if (!encode_out(&tout, type, (uint32_t)esize, C, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ldc, 1))
+      if (!encode_out(&tout, type, (uint32_t)esize, C, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ldc, 1,
+                      pl.v.tma_out == 2 ? 16 : 32))
         return GEMM_ERR_CUDA;
       p.out_tma = kOutTmaC;
     }

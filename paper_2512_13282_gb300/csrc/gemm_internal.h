@@ -53,7 +53,7 @@ struct TcVariant {
   bool b_kmajor; // B stored N x K (K contiguous)
   int epi;       // kEpiBf16 or kEpiS32
   bool pair;     // CTA-pair kernel (256-row tiles, cta_group::2) or single CTA (128 rows)
-  bool tma_out;  // epilogue stores through shared memory and TMA (see the instantiation files)
+  int tma_out;   // epilogue output variant: 0 direct stores, 1 TMA via 4 KB blocks, 2 TMA via 1 KB bf16 blocks
 };
 
 // Launch the persistent tcgen05 GEMM kernel (gemm_tc_bf16.cu / gemm_tc_s32.cu).
@@ -61,9 +61,9 @@ cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUten
                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
-// Whether the bf16 variant of a tile width stores through TMA.
-bool tc_bf16_tma_out(int bn);
-bool tc2_bf16_tma_out(int bn);
+// Output variant (TcVariant::tma_out) of the bf16 kernel of a tile width.
+int tc_bf16_tma_out(int bn);
+int tc2_bf16_tma_out(int bn);
 // Number of CTA pairs that can be resident at once (0 if unknown).
 int pair_slots();
 // The CTA-pair kernel (gemm_tc2_bf16.cu / gemm_tc2_s32.cu); grid is even.

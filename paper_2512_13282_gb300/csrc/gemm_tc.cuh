@@ -81,7 +81,7 @@ __host__ __device__ constexpr uint32_t pow2_at_least(uint32_t x) {
   return p;
 }
 
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 struct TcCfg {
   // MMA N for M = 128 is a multiple of 16 up to 256; the epilogue moves 32
   // columns per TMEM load; an MN-major B tile is assembled from 64-wide boxes.
@@ -94,9 +94,10 @@ struct TcCfg {
   static constexpr int kThreads = (2 + EPI_WARPS) * 32;
   static constexpr int kColsPerThread = BN / (EPI_WARPS / 4);
   static_assert(kColsPerThread % 16 == 0, "epilogue chunks are 32 columns, plus one of 16");
-  // TMA_OUT: per epilogue warp, one 32 x 32 block of 32-bit words (int32
-  // results or split-K partials of either path; bf16 results use half of it)
-  static constexpr uint32_t kEpiWarpBytes = TMA_OUT ? 4096 : 0;
+  // TMA_OUT 1: per epilogue warp, one 32 x 32 block of 32-bit words (int32
+  // results or split-K partials of either path; bf16 results use half of
+  // it); TMA_OUT 2 (bf16 C only): a 1 KB block of 32 rows x 16 bf16
+  static constexpr uint32_t kEpiWarpBytes = TMA_OUT == 1 ? 4096 : TMA_OUT == 2 ? 1024 : 0;
   static constexpr uint32_t kEpiOffset = STAGES * kStageBytes;  // 1024-byte aligned
   static constexpr uint32_t kBarOffset = kEpiOffset + EPI_WARPS * kEpiWarpBytes;
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
@@ -293,6 +294,31 @@ __device__ __forceinline__ void tma_out_bf16x32(const CUtensorMap *tm, uint32_t 
   }
 }
 
+// bf16 results through a 1 KB block: the 32 columns go out as two 16-column
+// halves (32-byte rows, 32-byte swizzle: chunk j of row r lands at chunk
+// j ^ ((r / 4) % 2)), one after the other.
+__device__ __forceinline__ void tma_out_bf16x16x2(const CUtensorMap *tm, uint32_t buf, int lane,
+                                                  const uint32_t (&r)[32], int x, int y, int M, int N) {
+  uint32_t h[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) h[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+  const uint32_t sw = (lane >> 2) & 1;
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    if (lane == 0) bulk_wait_read_all();
+    __syncwarp();
+    st_shared_v4(buf + lane * 32 + ((0u ^ sw) << 4), h[8 * half], h[8 * half + 1], h[8 * half + 2], h[8 * half + 3]);
+    st_shared_v4(buf + lane * 32 + ((1u ^ sw) << 4), h[8 * half + 4], h[8 * half + 5], h[8 * half + 6],
+                 h[8 * half + 7]);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0 && y < M && x + 16 * half < N) {
+      tma_store_2d(tm, buf, x + 16 * half, y);
+      bulk_commit();
+    }
+  }
+}
+
 // Requantised int8-path results (int16 or int8 C): 32 int32 sums of a row
 // requantised and packed into 64-byte (int16; 64-byte swizzle) or 32-byte
 // (int8; 32-byte swizzle: chunk j of row r lands at chunk j ^ ((r / 4) % 2))
@@ -343,12 +369,12 @@ __device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
     tmem_ld_32x32b_x16(taddr, r);
 }
 
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmOut, const TcParams p) {
   using Cfg = TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>;
-  const int out_tma = TMA_OUT ? p.out_tma : (int)kOutDirect;
+  const int out_tma = TMA_OUT != 0 ? p.out_tma : (int)kOutDirect;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-byte alignment
@@ -598,10 +624,12 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
           tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
           const int x = col0 + c * 32;
-          if (out_tma == kOutTmaWs) {
+          if (TMA_OUT == 1 && out_tma == kOutTmaWs) {
             tma_out_words32<true>(&tmOut, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
-          } else if (out_tma == kOutTmaC) {
+          } else if (TMA_OUT == 1 && out_tma == kOutTmaC) {
             tma_out_bf16x32(&tmOut, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
+          } else if (TMA_OUT == 2 && out_tma == kOutTmaC) {
+            tma_out_bf16x16x2(&tmOut, ebuf, lane, r, x, y0, p.M, p.N);
           } else if (row_ok) {
             if (split)
               store_words<32>(wrow, x, p.N, ws_vec, r);

@@ -90,7 +90,7 @@ __device__ __forceinline__ void tc_commit_pair_multicast(uint32_t bar) {
       : "memory");
 }
 
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 struct Tc2Cfg {
   static constexpr int kHalfN = BN / 2;  // B extent (in N) each CTA loads
   static_assert(kHalfN % 16 == 0 && BN <= 256, "pair MMA N is a multiple of 32 up to 256");
@@ -103,7 +103,7 @@ struct Tc2Cfg {
   static constexpr int kEpiThreads = EPI_WARPS * 32;
   static constexpr int kColsPerThread = BN / (EPI_WARPS / 4);
   static_assert(kColsPerThread % 16 == 0, "epilogue chunks are 32 columns, plus one of 16");
-  static constexpr uint32_t kEpiWarpBytes = TMA_OUT ? 4096 : 0;  // one 32 x 32 block of 32-bit words
+  static constexpr uint32_t kEpiWarpBytes = TMA_OUT == 1 ? 4096 : TMA_OUT == 2 ? 1024 : 0;  // one 32 x 32 block of 32-bit words
   static constexpr uint32_t kEpiOffset = STAGES * kStageBytes;
   static constexpr uint32_t kBarOffset = kEpiOffset + EPI_WARPS * kEpiWarpBytes;
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
@@ -114,12 +114,12 @@ struct Tc2Cfg {
 
 // Launch with cluster dimensions (2,1,1) and an even grid; tiles_m counts
 // 256-row tiles.
-template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, bool TMA_OUT>
+template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>::kThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmOut, const TcParams p) {
   using Cfg = Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>;
-  const int out_tma = TMA_OUT ? p.out_tma : (int)kOutDirect;
+  const int out_tma = TMA_OUT != 0 ? p.out_tma : (int)kOutDirect;
   constexpr int kTileM = 2 * kBM;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -379,10 +379,12 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
           tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
           const int x = col0 + c * 32;
-          if (out_tma == kOutTmaWs) {
+          if (TMA_OUT == 1 && out_tma == kOutTmaWs) {
             tma_out_words32<true>(&tmOut, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
-          } else if (out_tma == kOutTmaC) {
+          } else if (TMA_OUT == 1 && out_tma == kOutTmaC) {
             tma_out_bf16x32(&tmOut, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
+          } else if (TMA_OUT == 2 && out_tma == kOutTmaC) {
+            tma_out_bf16x16x2(&tmOut, ebuf, lane, r, x, y0, p.M, p.N);
           } else if (row_ok) {
             if (split)
               store_words<32>(wrow, x, p.N, ws_vec, r);

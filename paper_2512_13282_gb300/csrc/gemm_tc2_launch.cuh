@@ -6,7 +6,7 @@
 
 namespace gb300 {
 
-template <int BN, int STAGES, bool KM, int EPI, int EW, bool TMA>
+template <int BN, int STAGES, bool KM, int EPI, int EW, int TMA>
 cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
                         int grid,
                         cudaStream_t st) {

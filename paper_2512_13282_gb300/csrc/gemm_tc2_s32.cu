@@ -8,20 +8,20 @@ namespace gb300 {
 
 cudaError_t launch_tc2_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
-  const bool t = v.tma_out;
+  const bool t = v.tma_out != 0;
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_pair<256, 6, true, kEpiS32, 8, true>(a, b, o, p, grid, st);
-      case 224: return t ? launch_pair<224, 6, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
-                         : launch_pair<224, 7, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
-      case 192: return t ? launch_pair<192, 6, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
-                         : launch_pair<192, 7, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
-      case 128: return launch_pair<128, 8, true, kEpiS32, 4, true>(a, b, o, p, grid, st);
+      case 256: return launch_pair<256, 6, true, kEpiS32, 8, 1>(a, b, o, p, grid, st);
+      case 224: return t ? launch_pair<224, 6, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+                         : launch_pair<224, 7, true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+      case 192: return t ? launch_pair<192, 6, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+                         : launch_pair<192, 7, true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+      case 128: return launch_pair<128, 8, true, kEpiS32, 4, 1>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_pair<256, 6, false, kEpiS32, 8, true>(a, b, o, p, grid, st);
-      case 128: return launch_pair<128, 8, false, kEpiS32, 4, true>(a, b, o, p, grid, st);
+      case 256: return launch_pair<256, 6, false, kEpiS32, 8, 1>(a, b, o, p, grid, st);
+      case 128: return launch_pair<128, 8, false, kEpiS32, 4, 1>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;

@@ -4,7 +4,7 @@
 namespace gb300 {
 
 namespace {
-template <int BN, int STAGES, bool KM, int EPI, int EW, bool TMA>
+template <int BN, int STAGES, bool KM, int EPI, int EW, int TMA>
 cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
                        int grid,
                        cudaStream_t st) {
@@ -25,29 +25,31 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 }  // namespace
 
 // Tile widths compiled for the bf16 epilogue, with their stage counts and
-// output path (TMA stores through four 4 KB staging blocks, or direct
-// stores where the staging blocks would cost a pipeline stage): 128 (6,
-// TMA), 192 (5, TMA), 224 (5, direct; B column-major only), 256 (4, TMA).
+// output path (TMA stores through four 4 KB staging blocks, or, where those
+// would cost a pipeline stage, through four 1 KB blocks of 16 columns):
+// 128 (6, 4 KB), 192 (5, 4 KB), 224 (5, 1 KB; B column-major only), 256
+// (4, 4 KB).
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_one<256, 4, true, kEpiBf16, 4, true>(a, b, o, p, grid, st);
-      case 224: return launch_one<224, 5, true, kEpiBf16, 4, false>(a, b, o, p, grid, st);
-      case 192: return launch_one<192, 5, true, kEpiBf16, 4, true>(a, b, o, p, grid, st);
-      case 128: return launch_one<128, 6, true, kEpiBf16, 4, true>(a, b, o, p, grid, st);
+      case 256: return launch_one<256, 4, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 224: return launch_one<224, 5, true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
+      case 192: return launch_one<192, 5, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 128: return launch_one<128, 6, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_one<256, 4, false, kEpiBf16, 4, true>(a, b, o, p, grid, st);
-      case 192: return launch_one<192, 5, false, kEpiBf16, 4, true>(a, b, o, p, grid, st);
-      case 128: return launch_one<128, 6, false, kEpiBf16, 4, true>(a, b, o, p, grid, st);
+      case 256: return launch_one<256, 4, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 192: return launch_one<192, 5, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 128: return launch_one<128, 6, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;
 }
 
-// Whether launch_tc_bf16's variant for this tile width stores through TMA.
-bool tc_bf16_tma_out(int bn) { return bn != 224; }
+// Output variant (1: 4 KB TMA staging blocks, 2: 1 KB) of launch_tc_bf16's
+// kernel for this tile width.
+int tc_bf16_tma_out(int bn) { return bn == 224 ? 2 : 1; }
 
 }  // namespace gb300

@@ -4,7 +4,7 @@
 namespace gb300 {
 
 namespace {
-template <int BN, int STAGES, bool KM, int EPI, int EW, bool TMA>
+template <int BN, int STAGES, bool KM, int EPI, int EW, int TMA>
 cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
                        int grid,
                        cudaStream_t st) {
@@ -32,22 +32,22 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 // long reductions prefer (the planner's choice, v.tma_out).
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
-  const bool km = v.b_kmajor, t = v.tma_out;
+  const bool km = v.b_kmajor, t = v.tma_out != 0;
   switch (v.bn) {
-    case 256: return km ? launch_one<256, 4, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
-                        : launch_one<256, 4, false, kEpiS32, 8, true>(a, b, o, p, grid, st);
+    case 256: return km ? launch_one<256, 4, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+                        : launch_one<256, 4, false, kEpiS32, 8, 1>(a, b, o, p, grid, st);
     case 224:
       if (!km) return cudaErrorInvalidValue;
-      return t ? launch_one<224, 4, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
-               : launch_one<224, 5, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
+      return t ? launch_one<224, 4, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+               : launch_one<224, 5, true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
     case 192:
       if (km)
-        return t ? launch_one<192, 4, true, kEpiS32, 8, true>(a, b, o, p, grid, st)
-                 : launch_one<192, 5, true, kEpiS32, 8, false>(a, b, o, p, grid, st);
-      return t ? launch_one<192, 4, false, kEpiS32, 8, true>(a, b, o, p, grid, st)
-               : launch_one<192, 5, false, kEpiS32, 8, false>(a, b, o, p, grid, st);
-    case 128: return km ? launch_one<128, 6, true, kEpiS32, 4, true>(a, b, o, p, grid, st)
-                        : launch_one<128, 6, false, kEpiS32, 4, true>(a, b, o, p, grid, st);
+        return t ? launch_one<192, 4, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+                 : launch_one<192, 5, true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+      return t ? launch_one<192, 4, false, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+               : launch_one<192, 5, false, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+    case 128: return km ? launch_one<128, 6, true, kEpiS32, 4, 1>(a, b, o, p, grid, st)
+                        : launch_one<128, 6, false, kEpiS32, 4, 1>(a, b, o, p, grid, st);
   }
   return cudaErrorInvalidValue;
 }
