@@ -157,3 +157,35 @@ def test_requant_consistent_with_int32_path():
     for out, shift in (("int8_int16", 4), ("int8_int8", 12)):
         C = U.run(out, A, B, COL, shift=shift)
         assert np.array_equal(C.astype(np.int64), oracle.requantize(C32.astype(np.int64), shift, BITS[out]))
+
+
+DIRECT_CASES = [(300, 700, 1500, "1", None, 0), (130, 450, 3000, "3", None, 0), (300, 517, 640, "1", 523, 1),
+                (257, 333, 2100, "2", None, 0)]
+DIRECT_KERNELS = [(192, "0", ROW), (192, "0", COL), (224, "0", COL), (192, "1", COL), (224, "1", COL),
+                  (128, "0", COL), (256, "1", ROW)]
+
+
+@pytest.mark.parametrize("out", ["int8", "int8_int16", "int8_int8"])
+@pytest.mark.parametrize("bn,pair,layout", DIRECT_KERNELS,
+                         ids=[f"{b}-{'pair' if p == '1' else 'single'}-{'Brow' if l == ROW else 'Bcol'}"
+                              for b, p, l in DIRECT_KERNELS])
+def test_int8_direct_stores(out, bn, pair, layout, monkeypatch):
+    """The int8 epilogue without TMA stores (the direct-store kernels with
+    the extra pipeline stage at 192 / 224, the TMA kernels' fallback at 128 /
+    256): int32 and requantised C, split-K partials (including a pitch N that
+    is not a multiple of 4), ragged edges and unaligned C rows."""
+    monkeypatch.setenv("GB300_GEMM_TMA_STORE", "0")
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    monkeypatch.setenv("GB300_GEMM_BN", str(bn))
+    monkeypatch.setenv("GB300_GEMM_PAIR", pair)
+    for (M, N, K, splits, ldc, c_off) in DIRECT_CASES:
+        monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
+        A, B = _inputs(M, N, K, layout, seed=M + N + bn)
+        if out == "int8":
+            C = U.run(out, A, B, layout, ldc=ldc, c_off=c_off)
+            want = oracle.gemm_s8(A, B, layout)
+            assert np.array_equal(C.astype(np.int64), want), (M, N, K, splits)
+        else:
+            shift = _shift_for(out, K)
+            C = U.run(out, A, B, layout, ldc=ldc, c_off=c_off, shift=shift)
+            _check(out, A, B, layout, shift, C)
