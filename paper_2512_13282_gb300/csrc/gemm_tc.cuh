@@ -137,15 +137,27 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 // Reduced-precision int8 outputs (Sec. 5.1 reduces int8 GEMM outputs to 16
 // and 8 bits): the exact sum divided by 2^shift, rounded to nearest with
-// ties to even, saturated to [lo, hi].  shift is 0..31; a >> shift is the
-// floor (arithmetic shift) and r the non-negative remainder.
-__host__ __device__ __forceinline__ int32_t requantize_s32(int32_t a, int shift, int32_t lo, int32_t hi) {
-  int32_t q = a >> shift;
-  if (shift > 0) {
-    const uint32_t r = static_cast<uint32_t>(a) & ((1u << shift) - 1u);
-    const uint32_t half = 1u << (shift - 1);
-    q += (r > half || (r == half && (q & 1))) ? 1 : 0;  // |q| < 2^30 here: no overflow
+// ties to even, saturated to the output type.  RneShift does the division
+// and rounding in 32-bit arithmetic: q0 = a >> shift is the floor, r the
+// non-negative remainder a mod 2^shift, and (r + (q0 odd) + 2^(shift-1) - 1)
+// >> shift is 1 exactly when r > 2^(shift-1), or r = 2^(shift-1) with q0
+// odd; that sum stays below 2^32 for every shift 0..31.  With shift 0 all
+// terms but q0 vanish.
+struct RneShift {
+  int shift;
+  uint32_t mask, odd, half_m1;
+  __host__ __device__ explicit RneShift(int s)
+      : shift(s), mask(s ? (1u << s) - 1u : 0u), odd(s ? 1u : 0u), half_m1(s ? (1u << (s - 1)) - 1u : 0u) {}
+  __host__ __device__ __forceinline__ int32_t operator()(int32_t a) const {
+    const int32_t q0 = a >> shift;
+    const uint32_t t = (static_cast<uint32_t>(a) & mask) + (static_cast<uint32_t>(q0) & odd) + half_m1;
+    return q0 + static_cast<int32_t>(t >> shift);
   }
+};
+
+// The same, saturated to [lo, hi].
+__host__ __device__ __forceinline__ int32_t requantize_s32(int32_t a, int shift, int32_t lo, int32_t hi) {
+  const int32_t q = RneShift(shift)(a);
   return q < lo ? lo : (q > hi ? hi : q);
 }
 
@@ -325,20 +337,17 @@ __device__ __forceinline__ void tma_out_bf16x16x2(const CUtensorMap *tm, uint32_
 // rows, then stored like the other blocks.
 __device__ __forceinline__ void tma_out_narrow(const CUtensorMap *tm, uint32_t buf, int lane, const uint32_t (&v)[32],
                                                int bits, int shift, int x, int y, bool in_range) {
-  const int32_t hi = (1 << (bits - 1)) - 1, lo = -hi - 1;
+  // rounding in 32-bit arithmetic, saturation and packing by cvt.pack.sat
+  const RneShift rq(shift);
   uint32_t h[16];
   if (bits == 16) {
 #pragma unroll
-    for (int i = 0; i < 16; ++i)
-      h[i] = ((uint32_t)requantize_s32((int32_t)v[2 * i], shift, lo, hi) & 0xFFFFu) |
-             ((uint32_t)requantize_s32((int32_t)v[2 * i + 1], shift, lo, hi) << 16);
+    for (int i = 0; i < 16; ++i) h[i] = pack_sat_s16x2(rq((int32_t)v[2 * i]), rq((int32_t)v[2 * i + 1]));
   } else {
 #pragma unroll
     for (int i = 0; i < 8; ++i)
-      h[i] = ((uint32_t)requantize_s32((int32_t)v[4 * i], shift, lo, hi) & 0xFFu) |
-             (((uint32_t)requantize_s32((int32_t)v[4 * i + 1], shift, lo, hi) & 0xFFu) << 8) |
-             (((uint32_t)requantize_s32((int32_t)v[4 * i + 2], shift, lo, hi) & 0xFFu) << 16) |
-             ((uint32_t)requantize_s32((int32_t)v[4 * i + 3], shift, lo, hi) << 24);
+      h[i] = pack_sat_s8x4(rq((int32_t)v[4 * i]), rq((int32_t)v[4 * i + 1]), rq((int32_t)v[4 * i + 2]),
+                           rq((int32_t)v[4 * i + 3]));
   }
   if (lane == 0) bulk_wait_read_all();
   __syncwarp();

@@ -138,6 +138,21 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+// Two int32 values saturated to int16 and packed: lo in bits 0..15, hi in
+// bits 16..31 (cvt.pack places its second source in the low half).
+__device__ __forceinline__ uint32_t pack_sat_s16x2(int32_t lo, int32_t hi) {
+  uint32_t d;
+  asm("cvt.pack.sat.s16.s32 %0, %1, %2;" : "=r"(d) : "r"(hi), "r"(lo));
+  return d;
+}
+// Four int32 values saturated to int8 and packed, v0 in bits 0..7 (each
+// cvt.pack fills the low 16 bits and copies the rest from its third source).
+__device__ __forceinline__ uint32_t pack_sat_s8x4(int32_t v0, int32_t v1, int32_t v2, int32_t v3) {
+  uint32_t t, d;
+  asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(t) : "r"(v3), "r"(v2), "r"(0));
+  asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(v1), "r"(v0), "r"(t));
+  return d;
+}
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
