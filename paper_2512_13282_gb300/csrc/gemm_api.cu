@@ -109,8 +109,12 @@ gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
   return GEMM_OK;
 }
 
-// Test and benchmark overrides of the planner: GB300_GEMM_BN (128 or 256)
-// forces the tile width, GB300_GEMM_SPLITS (>= 1) the split-K factor.
+// Test and benchmark overrides of the planner, read at every call:
+// GB300_GEMM_BN (128, 192, 224 or 256) forces the tile width,
+// GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
+// split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
+// CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores, GB300_GEMM_PDL=0
+// plain stream ordering; GB300_GEMM_DEBUG=1 (read once) prints each plan.
 int env_int(const char *name) {
   const char *s = std::getenv(name);
   return s ? std::atoi(s) : 0;
