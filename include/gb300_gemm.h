@@ -28,13 +28,13 @@
  *     and split-K partials), allocated stream-ordered on first need and
  *     released by gemm_release_resources().  Calls on different streams that
  *     both need the workspace must be ordered by the caller.
- *   - Environment variables that override the planner (for tests and
- *     benchmarks; results are identical either way): GB300_GEMM_BN,
+ *   - Environment variables that override the planner, for tests and
+ *     benchmarks (int8 results are identical either way; bf16 results may
+ *     differ in summation order, within the same accuracy): GB300_GEMM_BN,
  *     GB300_GEMM_PAIR, GB300_GEMM_SPLITS, GB300_GEMM_SKINNY_MAX_M,
- *     GB300_GEMM_TMA_STORE=0, GB300_GEMM_PDL=0 (read at every call);
- *     GB300_GEMM_WAIT_LIMIT_MS (read once) sets
- *     the bound on every device-side wait (default 2000 ms); GB300_GEMM_DEBUG=1
- *     prints each plan to stderr.
+ *     GB300_GEMM_TMA_STORE=0 and GB300_GEMM_PDL=0, read at every call.
+ *     GB300_GEMM_WAIT_LIMIT_MS (read once) bounds every device-side wait
+ *     (default 2000 ms); GB300_GEMM_DEBUG=1 prints each plan to stderr.
  */
 #ifndef GB300_GEMM_H
 #define GB300_GEMM_H
