@@ -12,7 +12,9 @@ GEMM is bracketed by CUDA events on its stream, so flushes are not timed.
   e2e         the same through the C ABI from pinned HOST buffers: per step,
               H2D copies of every A and B, the GEMMs, D2H of every C, all
               inside the timed region; copies run on two copy streams and
-              overlap the other GEMMs' kernels
+              overlap the other GEMMs' kernels, and a GEMM with a large C is
+              issued as row blocks (the same call on rows of A and C) so
+              that its results start down while later rows compute
   roofline    the dominant kernel (largest share of step time): the main
               kernel of one GEMM (tensor-core, or CUDA-core for tiny M), timed
               through the library's profiling events in a second pass of the
@@ -151,6 +153,33 @@ class GemmCase:
         if st != 0:
             raise RuntimeError(f"{g.name}: {self.G.gemm_status_string(st)}")
 
+    def row_blocks(self, min_bytes=128 << 20, block_bytes=16 << 20, max_blocks=8):
+        """Row ranges [r0, r1) of A and C for the host-buffer pass.  A C of
+        at least `min_bytes` (over 0.6 ms on the download link) goes in
+        blocks of about `block_bytes` (at most `max_blocks`, multiples of 256
+        rows), so that its first rows travel back while later rows are
+        computed; smaller ones stay whole, since each block costs a launch
+        and, for int8, staging B again (measured: blocking the 4096^3 GEMMs
+        made the square sweep's host-buffer pass slower, the 8192^3 ones
+        made theirs faster)."""
+        M = self.g.M
+        if self.d2h < min_bytes:
+            return [(0, M)]
+        k = max(1, min(max_blocks, self.d2h // block_bytes))
+        rows = -(-M // k)
+        rows = -(-rows // 256) * 256
+        return [(r0, min(M, r0 + rows)) for r0 in range(0, M, rows)]
+
+    def launch_rows(self, r0, r1):
+        """The GEMM restricted to rows [r0, r1) of A and C (the same call on
+        a sub-matrix: A and C advance by whole rows, B is shared)."""
+        g = self.g
+        pa = self.A.data_ptr() + r0 * g.K * self.A.element_size()
+        pc = self.C.data_ptr() + r0 * g.N * self.C.element_size()
+        st = self.fn(r1 - r0, g.N, g.K, pa, g.K, self.B, self.ldb, g.layout, pc, g.N, None)
+        if st != 0:
+            raise RuntimeError(f"{g.name} rows {r0}..{r1}: {self.G.gemm_status_string(st)}")
+
     def launch_e2e(self):
         self.A.copy_(self.hA, non_blocking=True)
         self.B.copy_(self.hB, non_blocking=True)
@@ -252,28 +281,40 @@ def run_ours(args, rank, world, dev):
         by_size = sorted(cases, key=lambda c: c.h2d + c.d2h)
         e2e_cases = by_size[0::2] + by_size[1::2][::-1]
 
+        # A GEMM whose C is large goes as row blocks (B once, then A rows,
+        # the call on those rows, their C rows back): its first results
+        # travel down while the later blocks still compute.  The views and
+        # events are made once, so that a step only enqueues work.
+        plan = []  # per GEMM: (case, B copy, [(A rows copy, C rows copy, r0, r1, uploaded, done)])
+        for c in e2e_cases:
+            bl = c.row_blocks()
+            whole = len(bl) == 1
+            items = [(c.A[r0:r1], c.hA[r0:r1], c.hC[r0:r1], c.C[r0:r1], None if whole else (r0, r1),
+                      torch.cuda.Event(), torch.cuda.Event()) for (r0, r1) in bl]
+            plan.append((c, items))
+
         def e2e_step(start, stop):
             start.record(stream)
             h2d.wait_stream(stream)
-            up = []
             with torch.cuda.stream(h2d):
-                for c in e2e_cases:
-                    c.A.copy_(c.hA, non_blocking=True)
+                for c, items in plan:
                     c.B.copy_(c.hB, non_blocking=True)
-                    e = torch.cuda.Event()
-                    e.record(h2d)
-                    up.append(e)
-            done = []
-            for c, e in zip(e2e_cases, up):
-                stream.wait_event(e)
-                c.launch()
-                e2 = torch.cuda.Event()
-                e2.record(stream)
-                done.append(e2)
+                    for (da, ha, hc, dc, rows, up, done) in items:
+                        da.copy_(ha, non_blocking=True)
+                        up.record(h2d)
+            for c, items in plan:
+                for (da, ha, hc, dc, rows, up, done) in items:
+                    stream.wait_event(up)
+                    if rows is None:
+                        c.launch()
+                    else:
+                        c.launch_rows(*rows)
+                    done.record(stream)
             with torch.cuda.stream(d2h):
-                for c, e2 in zip(e2e_cases, done):
-                    d2h.wait_event(e2)
-                    c.hC.copy_(c.C, non_blocking=True)
+                for c, items in plan:
+                    for (da, ha, hc, dc, rows, up, done) in items:
+                        d2h.wait_event(done)
+                        hc.copy_(dc, non_blocking=True)
             stream.wait_stream(d2h)
             stop.record(stream)
 
@@ -282,12 +323,33 @@ def run_ours(args, rank, world, dev):
         torch.cuda.synchronize()
         e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(args.steps)]
+        issue_s = []
         for k in range(args.steps):
             flush.fill_(float(k))
             torch.cuda.synchronize()
+            t0 = time.perf_counter()
             e2e_step(*e_ev[k])
+            issue_s.append(time.perf_counter() - t0)
         torch.cuda.synchronize()
         e2e_ms = sum(a.elapsed_time(b) for a, b in e_ev) / args.steps
+        if rank == 0:
+            print(f"e2e: {e2e_ms:.3f} ms per step on the device clock, {1e3 * statistics.median(issue_s):.3f} ms "
+                  "to issue a step on the host", file=sys.stderr)
+        # The results that came back through the row blocks equal those of
+        # one whole-matrix call (int8: bit for bit; bf16: the blocks may
+        # split K differently, so within a bf16 rounding step).
+        for c in e2e_cases:
+            c.launch()
+            whole = c.C.cpu()
+            got = c.hC.clone()
+            if c.g.dtype == "bf16":
+                a = whole.view(torch.bfloat16).float()
+                b = got.view(torch.bfloat16).float()
+                ok = bool(torch.all((a - b).abs() <= 2.0 ** -7 * torch.maximum(a.abs(), b.abs())))
+            else:
+                ok = torch.equal(whole, got)
+            if not ok:
+                raise RuntimeError(f"{c.g.name}: host-buffer results differ from the whole-matrix call")
 
     # max over ranks
     vals = torch.tensor([gemm_ms, e2e_ms or 0.0, wall], dtype=torch.float64, device=dev)

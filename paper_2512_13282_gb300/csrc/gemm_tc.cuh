@@ -14,19 +14,20 @@
 //                      into one of two TMEM accumulators; the first MMA of a
 //                      tile overwrites instead of accumulating, which takes
 //                      the place of the paper's zeroing kernel (Sec. 4.2.1).
-//   warps 2..          epilogue: TMEM -> registers -> bf16 (RNE) or int32 ->
-//                      a 32-row x 32-column block in the warp's own shared
-//                      memory (swizzled as the TMA expects) -> one TMA tensor
-//                      store per block, which writes whole lines of C and
-//                      clips at the M/N edges (stores that each lane makes to
-//                      its own row would touch 32 lines per instruction and
-//                      compete with the operand traffic; where C's address
-//                      or pitch rules TMA out, lanes store their rows
-//                      directly).  Two
-//                      accumulators let the epilogue of one tile overlap the
-//                      main loop of the next (the paper keeps a single C
-//                      buffer for lack of L1 space, Sec. 5.3.2; TMEM has room
-//                      for two).
+//   warps 2..          epilogue: TMEM -> registers -> bf16 (RNE), int32, or
+//                      int32 requantised to int16 / int8 -> a 32-row block
+//                      in the warp's own shared memory (swizzled as the TMA
+//                      expects) -> one TMA tensor store per block, which
+//                      writes whole lines of C and clips at the M/N edges.
+//                      Stores that each lane makes to its own row touch 32
+//                      lines per instruction and compete with the operand
+//                      traffic; lanes store their rows directly only where
+//                      C's address or pitch rules TMA out, and in the int8
+//                      variants that trade the staging blocks for a pipeline
+//                      stage (long reductions).  Two accumulators let the
+//                      epilogue of one tile overlap the main loop of the
+//                      next (the paper keeps a single C buffer for lack of
+//                      L1 space, Sec. 5.3.2; TMEM has room for two).
 //
 // Exact int8 emulation (kEpiS32): int8 operands, staged as bf16 (every int8
 // value is exact in bf16), are multiplied on the bf16 pipe.  A product is at
