@@ -25,25 +25,6 @@ __device__ __forceinline__ uint32_t s8_to_bf16_bits(int v) {
   return __float_as_uint(static_cast<float>(v)) >> 16;
 }
 
-// Four int8 (byte i of w is element i) -> four bf16 bit patterns, elements
-// 0, 1 in lo and 2, 3 in hi (element 2i in the low half).  Without the
-// quarter-rate int -> float conversion: byte b, flipped to b + 128 in
-// 0..255, becomes the low mantissa byte of the float 2^23, i.e. the float
-// 2^23 + b + 128, and subtracting 2^23 + 128 leaves b exactly (integers
-// below 2^24 are exact in fp32, so is their difference).  The float's upper
-// half is then the bf16 of b, as above.
-__device__ __forceinline__ void s8x4_to_bf16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
-  constexpr uint32_t kTwo23 = 0x4B000000u;  // 2^23
-  constexpr float kBias = 8388736.0f;       // 2^23 + 128
-  const uint32_t u = w ^ 0x80808080u;
-  const uint32_t f0 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7650)), kBias));
-  const uint32_t f1 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7651)), kBias));
-  const uint32_t f2 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7652)), kBias));
-  const uint32_t f3 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7653)), kBias));
-  lo = __byte_perm(f0, f1, 0x7632);  // upper halves: element 0 low, element 1 high
-  hi = __byte_perm(f2, f3, 0x7632);
-}
-
 // Converts 16 int8 held in a uint4 to 16 bf16 bit patterns in two uint4.
 __device__ __forceinline__ void s8x16_to_bf16x16(const int4 raw, uint4 &lo, uint4 &hi) {
   uint32_t o[8];

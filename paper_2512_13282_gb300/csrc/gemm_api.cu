@@ -505,6 +505,121 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
 
 namespace {
 
+// int8 operand streamed by gemm_s8tm_kernel: K-contiguous rows, boxes of
+// 128 bytes x 128 rows with the 128-byte swizzle its converter warps expect.
+bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t K, uint64_t rows, uint64_t ld) {
+  const cuuint64_t dims[2] = {K, rows};
+  const cuuint64_t strides[1] = {ld};
+  const cuuint32_t box[2] = {128, (cuuint32_t)kBM};
+  const cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Memory-bound int8 shapes, where one operand is far larger than the other:
+// M <= 128 with B stored N x K (the weights, P = B, are streamed as int8 and
+// the activations Q = A staged), or N <= 128 with M > 128 (P = A, Q = B).
+// gemm_s8tm_kernel converts P inside the kernel, so P moves once as int8
+// instead of three times as staged bf16.  Returns false, having launched
+// nothing, when the shape or P's alignment (16-byte base and pitch, for
+// TMA) rules the path out; GB300_GEMM_S8TM=0 turns it off and
+// GB300_GEMM_SPLITS forces the split-K factor.
+bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda, const int8_t *B,
+              int64_t ldb, bool b_kmajor, void *C, int64_t ldc, int out_bits, int shift, cudaStream_t st,
+              gemm_status_t *status) {
+  const char *env = std::getenv("GB300_GEMM_S8TM");
+  if (env && std::atoi(env) == 0) return false;
+  bool swap;
+  if (b_kmajor && M <= kBM && N > kBM)
+    swap = true;
+  else if (N <= kBM && M > kBM)
+    swap = false;
+  else
+    return false;
+  const int8_t *P = swap ? B : A;
+  const int64_t ldp = swap ? ldb : lda;
+  if (!aligned16(P) || ldp % 16 != 0) return false;
+  const int64_t P_rows = swap ? N : M, Q_rows = swap ? M : N;
+  const int qn = Q_rows <= 64 ? 64 : 128;
+  // Q is staged as bf16 in its own layout: A (M x K) when swapped, else B.
+  const bool q_kmajor = swap || b_kmajor;
+  const int8_t *Qs = swap ? A : B;
+  const int64_t ldq_src = swap ? lda : ldb;
+  const int64_t q_st_rows = q_kmajor ? Q_rows : K, q_st_cols = q_kmajor ? K : Q_rows;
+  const int64_t ldq = (q_st_cols + 7) / 8 * 8;
+  const int64_t num_kb = ceil_div(K, kS8tmKB);
+  const int64_t tiles_p = ceil_div(P_rows, kBM), tiles_q = ceil_div(Q_rows, qn);
+  const int64_t tiles = tiles_p * tiles_q;
+  int64_t splits = (int64_t)d.sms / tiles;
+  if (splits > num_kb / 4) splits = num_kb / 4;
+  if (splits > 16) splits = 16;
+  if (splits < 1) splits = 1;
+  const int force_splits = env_int("GB300_GEMM_SPLITS");
+  if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
+  const int64_t kb_per = ceil_div(num_kb, splits);
+  splits = ceil_div(num_kb, kb_per);
+  gemm_status_t s;
+  const size_t q_bytes = align_up((size_t)q_st_rows * ldq * 2, 256);
+  const size_t total = q_bytes + (splits > 1 ? (size_t)splits * M * N * 4 : 0);
+  if ((s = ensure_workspace(d, total, st)) != GEMM_OK) {
+    *status = s;
+    return true;
+  }
+  uint8_t *ws = static_cast<uint8_t *>(d.ws);
+  uint16_t *Qb = reinterpret_cast<uint16_t *>(ws);
+  *status = GEMM_ERR_CUDA;
+  g_launches.fetch_add(1);
+  if (launch_s8_to_bf16_pair(S8Job{Qs, q_st_rows, q_st_cols, ldq_src, Qb, ldq},
+                             S8Job{nullptr, 0, 0, 0, nullptr, 0}, d.sms, st) != cudaSuccess)
+    return true;
+  CUtensorMap tp, tq;
+  if (!encode_s8_rows(&tp, P, (uint64_t)K, (uint64_t)P_rows, (uint64_t)ldp)) return true;
+  const bool ok_q = q_kmajor ? encode_bf16_2d(&tq, Qb, (uint64_t)K, (uint64_t)Q_rows, (uint64_t)ldq, kBK, qn)
+                             : encode_bf16_2d(&tq, Qb, (uint64_t)Q_rows, (uint64_t)K, (uint64_t)ldq, 64, kBK);
+  if (!ok_q) return true;
+  S8tmParams p{};
+  p.P_rows = (int)P_rows;
+  p.Q_rows = (int)Q_rows;
+  p.K = (int)K;
+  p.M = (int)M;
+  p.N = (int)N;
+  p.tiles_p = (int)tiles_p;
+  p.tiles_q = (int)tiles_q;
+  p.num_kb = (int)num_kb;
+  p.splits = (int)splits;
+  p.kb_per_split = (int)kb_per;
+  p.slab_kb = 1024 / kS8tmKB;
+  p.swap = swap ? 1 : 0;
+  p.C = C;
+  p.ldc = ldc;
+  p.ws = splits > 1 ? ws + q_bytes : nullptr;
+  p.err = d.err;
+  p.wait_limit_ns = wait_limit_ns();
+  p.out_bits = out_bits;
+  p.out_shift = shift;
+  const int64_t units = tiles * splits;
+  const int grid = (int)(units < d.sms ? units : d.sms);
+  static const bool debug = env_int("GB300_GEMM_DEBUG") != 0;
+  if (debug)
+    std::fprintf(stderr, "[gb300_gemm] M=%lld N=%lld K=%lld int8 s8tm %s QN=%d Q %s tiles=%lldx%lld splits=%lld grid=%d\n",
+                 (long long)M, (long long)N, (long long)K, swap ? "swap" : "direct", qn,
+                 q_kmajor ? "K-major" : "MN-major", (long long)tiles_p, (long long)tiles_q, (long long)splits, grid);
+  const bool prof = g_prof_start && g_prof_stop;
+  if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
+  g_launches.fetch_add(1);
+  if (launch_s8tm(qn, q_kmajor, tp, tq, p, grid, st) != cudaSuccess) return true;
+  if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
+  if (splits > 1) {
+    g_launches.fetch_add(1);
+    if (launch_splitk_reduce_s32(static_cast<const int32_t *>(p.ws), (int)splits, M, N, C, ldc, out_bits, shift,
+                                 d.sms, st) != cudaSuccess)
+      return true;
+  }
+  *status = GEMM_OK;
+  return true;
+}
+
 // The int8 GEMM behind gemm_s8s8_s32 (out_bits 32), gemm_s8s8_s16 and
 // gemm_s8s8_s8 (out_bits 16 / 8, right shift `shift`): the exact int32 sum
 // is formed the same way for all three; only the final store differs.
@@ -527,6 +642,7 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
   if (M <= skinny_max_m(true))
     return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, true, st, out_bits, shift);
+  if (try_s8tm(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, out_bits, shift, st, &s)) return s;
   Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
   pl.p.out_bits = out_bits;
   pl.p.out_shift = shift;

@@ -72,6 +72,32 @@ cudaError_t launch_tc2_bf16(const TcVariant &v, const CUtensorMap &a, const CUte
 cudaError_t launch_tc2_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
 
+// int8 GEMM for memory-bound shapes with the large operand converted to bf16
+// inside the kernel (gemm_s8tm.cu).  P (int8, K contiguous, P_rows x K) is
+// the operand streamed from HBM; Q (bf16, staged, Q_rows x K) the small
+// one.  The sum over k of P[p][k] * Q[q][k] is C[q][p] when swap (P = B
+// stored N x K, Q = A) and C[p][q] otherwise (P = A, Q = B).
+constexpr int kS8tmKB = 128;  // K per k-block of gemm_s8tm_kernel
+struct S8tmParams {
+  int P_rows, Q_rows, K;
+  int M, N;          // C extents
+  int tiles_p, tiles_q;
+  int num_kb;        // ceil(K / kS8tmKB)
+  int splits, kb_per_split;
+  int slab_kb;       // k-blocks per exact fp32 slab (1024 / kS8tmKB)
+  int swap;
+  void *C;
+  int64_t ldc;
+  void *ws;          // split-K partials: splits x M x N int32 (row pitch N)
+  uint32_t *err;
+  uint64_t wait_limit_ns;
+  int out_bits;      // 32, 16 or 8
+  int out_shift;
+};
+// qn: 64 or 128 columns of Q per tile; q_kmajor: Q stored Q_rows x K.
+cudaError_t launch_s8tm(int qn, bool q_kmajor, const CUtensorMap &tp, const CUtensorMap &tq, const S8tmParams &p,
+                        int grid, cudaStream_t st);
+
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
 // int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is
 // rows x cols with an arbitrary source leading dimension.

@@ -1,6 +1,7 @@
 // ptx.cuh -- thin inline-PTX wrappers for the sm_103a features the GEMM
 // kernels use: mbarriers, TMA tensor copies, and the 5th-generation tensor
-// core (tcgen05: TMEM allocation, MMA, commit, TMEM loads).  Encodings follow
+// core (tcgen05: TMEM allocation, MMA, commit, TMEM loads and stores); plus
+// the exact int8 -> bf16 conversion the int8 kernels share.  Encodings follow
 // the public PTX ISA (tcgen05 instruction descriptor and shared-memory matrix
 // descriptor tables).
 #pragma once
@@ -157,6 +158,28 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
+// ------------------------------------------------------------ int8 -> bf16
+
+// Four int8 (byte i of w is element i) -> four bf16 bit patterns, elements
+// 0, 1 in lo and 2, 3 in hi (element 2i in the low half).  Without the
+// quarter-rate int -> float conversion: byte b, flipped to b + 128 in
+// 0..255, becomes the low mantissa byte of the float 2^23, i.e. the float
+// 2^23 + b + 128, and subtracting 2^23 + 128 leaves b exactly (integers
+// below 2^24 are exact in fp32, so is their difference).  |b| <= 128 needs
+// at most 8 significant bits, which a bf16 has, so the float's upper half is
+// the exact bf16 of b.
+__device__ __forceinline__ void s8x4_to_bf16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+  constexpr uint32_t kTwo23 = 0x4B000000u;  // 2^23
+  constexpr float kBias = 8388736.0f;       // 2^23 + 128
+  const uint32_t u = w ^ 0x80808080u;
+  const uint32_t f0 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7650)), kBias));
+  const uint32_t f1 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7651)), kBias));
+  const uint32_t f2 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7652)), kBias));
+  const uint32_t f3 = __float_as_uint(__fsub_rn(__uint_as_float(__byte_perm(u, kTwo23, 0x7653)), kBias));
+  lo = __byte_perm(f0, f1, 0x7632);  // upper halves: element 0 low, element 1 high
+  hi = __byte_perm(f2, f3, 0x7632);
+}
+
 // ----------------------------------------------------------------- tcgen05
 
 template <uint32_t kCols>
@@ -188,6 +211,19 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, ui
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem], kind::f16: A is 128 rows (TMEM lanes) of
+// K = 16 bf16 packed two to a 32-bit column (the lower k in the low half),
+// i.e. 8 columns starting at a_tmem.
+__device__ __forceinline__ void tc_mma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                                   uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 
@@ -245,6 +281,43 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&r)
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr)
       : "memory");
+}
+
+// Thread t of the warp writes r[0..31] to columns [col, col+32) of TMEM
+// lane (lane base + t).
+__device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+      "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+      "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+// Thread t of the warp writes r[0..63] to columns [col, col+64) of TMEM
+// lane (lane base + t).
+__device__ __forceinline__ void tmem_st_32x32b_x64(uint32_t taddr, const uint32_t (&r)[64]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31]), "r"(r[32]), "r"(r[33]), "r"(r[34]), "r"(r[35]), "r"(r[36]), "r"(r[37]), "r"(r[38]), "r"(r[39]), "r"(r[40]), "r"(r[41]), "r"(r[42]), "r"(r[43]), "r"(r[44]), "r"(r[45]), "r"(r[46]), "r"(r[47]), "r"(r[48]), "r"(r[49]), "r"(r[50]), "r"(r[51]), "r"(r[52]), "r"(r[53]), "r"(r[54]), "r"(r[55]), "r"(r[56]), "r"(r[57]), "r"(r[58]), "r"(r[59]), "r"(r[60]), "r"(r[61]), "r"(r[62]), "r"(r[63])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
 }
 
 __device__ __forceinline__ void tmem_ld_wait() {

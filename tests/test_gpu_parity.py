@@ -332,3 +332,69 @@ def test_int8_back_to_back_calls(monkeypatch):
     assert G.gemm_device_status() == G.GEMM_OK
     for A, B, layout, _, _, C in keep:
         _check("int8", A, B, layout, C.cpu().numpy())
+
+
+# ------------------------ int8 with the large operand converted in the kernel
+
+S8TM = [
+    # M <= 128, B stored N x K: the weights are streamed as int8 (swap)
+    (16, 512, 4096, COL), (128, 4096, 1000, COL), (100, 1000, 3000, COL), (64, 300, 64, COL),
+    (9, 129, 1024, COL), (128, 1500, 8192, COL),
+    # N <= 128, M > 128: A is streamed as int8, B (either layout) staged
+    (1000, 64, 3008, ROW), (300, 128, 4096, COL), (2000, 17, 1024, ROW), (129, 100, 2048, COL),
+    (640, 65, 11008, ROW),
+]
+
+
+@pytest.mark.parametrize("M,N,K,layout", S8TM, ids=[f"{m}x{n}x{k}-{'Bcol' if l else 'Brow'}"
+                                                    for m, n, k, l in S8TM])
+@pytest.mark.parametrize("splits", ["auto", "1", "3"])
+def test_int8_converted_in_kernel(M, N, K, layout, splits, monkeypatch):
+    """The int8 kernel that converts its large operand to bf16 in tensor
+    memory (swap for small M, direct for small N): ragged tiles in every
+    dimension, forced split-K, bit-exact against the oracle."""
+    if splits != "auto":
+        monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
+    A, B = _inputs("int8", M, N, K, layout, seed=M * 5 + N + K)
+    C = U.run("int8", A, B, layout)
+    _check("int8", A, B, layout, C)
+
+
+@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (300, 128, 4096, ROW)], ids=["swap", "direct"])
+@pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
+@pytest.mark.parametrize("shift", [0, 7, 12])
+def test_int8_converted_in_kernel_requantised(M, N, K, layout, out, shift):
+    A, B = _inputs("int8", M, N, K, layout, seed=shift + M)
+    C = U.run(out, A, B, layout, shift=shift)
+    want = oracle.requantize(oracle.gemm_s8(A, B, layout), shift, 16 if out == "int8_int16" else 8)
+    assert np.array_equal(C.astype(np.int64), want)
+
+
+def test_int8_converted_in_kernel_extremes(monkeypatch):
+    """All -128 (every 1024-deep slab is exactly 2^24), the largest exact K,
+    and M = 1 on this path (the CUDA-core kernel turned off)."""
+    A = np.full((128, 4096), -128, np.int8)
+    B = np.full((300, 4096), -128, np.int8)
+    assert (U.run("int8", A, B, COL) == 16384 * 4096).all()
+    A = np.full((16, 131071), -128, np.int8)
+    B = np.full((200, 131071), -128, np.int8)
+    assert (U.run("int8", A, B, COL) == 2147467264).all()
+    B[:, :] = 127
+    assert (U.run("int8", A, B, COL) == -16256 * 131071).all()
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    A1, B1 = _inputs("int8", 1, 700, 640, COL, seed=3)
+    _check("int8", A1, B1, COL, U.run("int8", A1, B1, COL))
+
+
+@pytest.mark.parametrize("M,N,K,layout", [(128, 4096, 4096, COL), (8192, 64, 8192, ROW)], ids=["swap", "direct"])
+def test_int8_converted_in_kernel_matches_general_path(M, N, K, layout, monkeypatch):
+    """Full-size shapes of the benchmark: the new path and the general
+    (staged) path give the same int32 results, and sampled entries match the
+    oracle."""
+    A, B = _inputs("int8", M, N, K, layout, seed=7)
+    C1 = U.run("int8", A, B, layout)
+    monkeypatch.setenv("GB300_GEMM_S8TM", "0")
+    C0 = U.run("int8", A, B, layout)
+    assert np.array_equal(C0, C1)
+    r, c = _sample_positions(M, N, seed=3)
+    assert np.array_equal(C1[r, c].astype(np.int64), oracle.gemm_s8_entries(A, B, layout, r, c))
