@@ -519,7 +519,8 @@ bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t K, uint64_t row
 
 // Memory-bound int8 shapes, where one operand is far larger than the other:
 // M <= 128 with B stored N x K (the weights, P = B, are streamed as int8 and
-// the activations Q = A staged), or N <= 128 with M > 128 (P = A, Q = B).
+// the activations Q = A staged), or N <= 128 with M > 128 (P = A, Q = B, in
+// either layout).
 // gemm_s8tm_kernel converts P inside the kernel, so P moves once as int8
 // instead of three times as staged bf16.  Returns false, having launched
 // nothing, when the shape or P's alignment (16-byte base and pitch, for
@@ -542,12 +543,10 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   if (!aligned16(P) || ldp % 16 != 0) return false;
   const int64_t P_rows = swap ? N : M, Q_rows = swap ? M : N;
   const int qn = Q_rows <= 64 ? 64 : 128;
-  // Q is staged as bf16 in its own layout: A (M x K) when swapped, else B.
-  const bool q_kmajor = swap || b_kmajor;
+  // Q(q, k): A[q][k] when swapped; else B, stored N x K or K x N.
   const int8_t *Qs = swap ? A : B;
-  const int64_t ldq_src = swap ? lda : ldb;
-  const int64_t q_st_rows = q_kmajor ? Q_rows : K, q_st_cols = q_kmajor ? K : Q_rows;
-  const int64_t ldq = (q_st_cols + 7) / 8 * 8;
+  const int64_t sq = (swap || b_kmajor) ? (swap ? lda : ldb) : 1;
+  const int64_t sk = (swap || b_kmajor) ? 1 : ldb;
   const int64_t num_kb = ceil_div(K, kS8tmKB);
   const int64_t tiles_p = ceil_div(P_rows, kBM), tiles_q = ceil_div(Q_rows, qn);
   const int64_t tiles = tiles_p * tiles_q;
@@ -560,24 +559,18 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   const int64_t kb_per = ceil_div(num_kb, splits);
   splits = ceil_div(num_kb, kb_per);
   gemm_status_t s;
-  const size_t q_bytes = align_up((size_t)q_st_rows * ldq * 2, 256);
+  const size_t q_bytes = align_up(s8tm_q_image_bytes(qn, Q_rows, K), 256);
   const size_t total = q_bytes + (splits > 1 ? (size_t)splits * M * N * 4 : 0);
   if ((s = ensure_workspace(d, total, st)) != GEMM_OK) {
     *status = s;
     return true;
   }
   uint8_t *ws = static_cast<uint8_t *>(d.ws);
-  uint16_t *Qb = reinterpret_cast<uint16_t *>(ws);
   *status = GEMM_ERR_CUDA;
   g_launches.fetch_add(1);
-  if (launch_s8_to_bf16_pair(S8Job{Qs, q_st_rows, q_st_cols, ldq_src, Qb, ldq},
-                             S8Job{nullptr, 0, 0, 0, nullptr, 0}, d.sms, st) != cudaSuccess)
-    return true;
-  CUtensorMap tp, tq;
+  if (launch_s8tm_stage_q(Qs, sq, sk, Q_rows, K, qn, ws, st) != cudaSuccess) return true;
+  CUtensorMap tp;
   if (!encode_s8_rows(&tp, P, (uint64_t)K, (uint64_t)P_rows, (uint64_t)ldp)) return true;
-  const bool ok_q = q_kmajor ? encode_bf16_2d(&tq, Qb, (uint64_t)K, (uint64_t)Q_rows, (uint64_t)ldq, kBK, qn)
-                             : encode_bf16_2d(&tq, Qb, (uint64_t)Q_rows, (uint64_t)K, (uint64_t)ldq, 64, kBK);
-  if (!ok_q) return true;
   S8tmParams p{};
   p.P_rows = (int)P_rows;
   p.Q_rows = (int)Q_rows;
@@ -598,17 +591,18 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   p.wait_limit_ns = wait_limit_ns();
   p.out_bits = out_bits;
   p.out_shift = shift;
+  p.q_img = ws;
   const int64_t units = tiles * splits;
   const int grid = (int)(units < d.sms ? units : d.sms);
   static const bool debug = env_int("GB300_GEMM_DEBUG") != 0;
   if (debug)
-    std::fprintf(stderr, "[gb300_gemm] M=%lld N=%lld K=%lld int8 s8tm %s QN=%d Q %s tiles=%lldx%lld splits=%lld grid=%d\n",
-                 (long long)M, (long long)N, (long long)K, swap ? "swap" : "direct", qn,
-                 q_kmajor ? "K-major" : "MN-major", (long long)tiles_p, (long long)tiles_q, (long long)splits, grid);
+    std::fprintf(stderr, "[gb300_gemm] M=%lld N=%lld K=%lld int8 s8tm %s QN=%d tiles=%lldx%lld splits=%lld grid=%d\n",
+                 (long long)M, (long long)N, (long long)K, swap ? "swap" : "direct", qn, (long long)tiles_p,
+                 (long long)tiles_q, (long long)splits, grid);
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
   g_launches.fetch_add(1);
-  if (launch_s8tm(qn, q_kmajor, tp, tq, p, grid, st) != cudaSuccess) return true;
+  if (launch_s8tm(qn, tp, p, grid, st) != cudaSuccess) return true;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
   if (splits > 1) {
     g_launches.fetch_add(1);

@@ -74,9 +74,10 @@ cudaError_t launch_tc2_s32(const TcVariant &v, const CUtensorMap &a, const CUten
 
 // int8 GEMM for memory-bound shapes with the large operand converted to bf16
 // inside the kernel (gemm_s8tm.cu).  P (int8, K contiguous, P_rows x K) is
-// the operand streamed from HBM; Q (bf16, staged, Q_rows x K) the small
-// one.  The sum over k of P[p][k] * Q[q][k] is C[q][p] when swap (P = B
-// stored N x K, Q = A) and C[p][q] otherwise (P = A, Q = B).
+// the operand streamed from HBM; Q (Q_rows x K) the small one, staged by
+// launch_s8tm_stage_q as bf16 shared-memory images.  The sum over k of
+// P[p][k] * Q[q][k] is C[q][p] when swap (P = B stored N x K, Q = A) and
+// C[p][q] otherwise (P = A, Q = B).
 constexpr int kS8tmKB = 128;  // K per k-block of gemm_s8tm_kernel
 struct S8tmParams {
   int P_rows, Q_rows, K;
@@ -93,10 +94,15 @@ struct S8tmParams {
   uint64_t wait_limit_ns;
   int out_bits;      // 32, 16 or 8
   int out_shift;
+  const void *q_img; // Q's images, tiles_q x num_kb of them (s8tm_q_image_bytes in all)
 };
-// qn: 64 or 128 columns of Q per tile; q_kmajor: Q stored Q_rows x K.
-cudaError_t launch_s8tm(int qn, bool q_kmajor, const CUtensorMap &tp, const CUtensorMap &tq, const S8tmParams &p,
-                        int grid, cudaStream_t st);
+// Bytes of Q's images for QN = qn columns per tile.
+size_t s8tm_q_image_bytes(int qn, int64_t Q_rows, int64_t K);
+// Writes Q's images: Q(q, k) = src[q * sq + k * sk] (int8), exact bf16.
+cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64_t Q_rows, int64_t K, int qn,
+                                void *img, cudaStream_t st);
+// qn: 64 or 128 columns of Q per tile.
+cudaError_t launch_s8tm(int qn, const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st);
 
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
 // int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is

@@ -13,18 +13,21 @@
 //   P  the large operand, int8, K contiguous: B stored N x K when M is
 //      small (P row = column n of C), or A when N is small (P row = row m).
 //      It is the MMA's 128-row A operand, read from TMEM.
-//   Q  the small operand, staged as bf16 beforehand (K-major or MN-major);
-//      the MMA's QN-column B operand, read from shared memory.
+//   Q  the small operand, staged beforehand (s8tm_stage_q_kernel) as the
+//      exact shared-memory image the MMA reads for each (Q tile, k-block):
+//      bf16, K-major, 128-byte swizzled, QN rows x 128 K = QN x 256 bytes,
+//      contiguous; zero outside the matrix.  It is the MMA's QN-column B
+//      operand.
 //
-// Roles (10 warps):
-//   warp 0 (one lane)  TMA producer: per k-block of 128 a 128 x 128 int8
-//                      box of P (128-byte rows, 128-byte swizzle) and two
-//                      QN x 64 bf16 boxes of Q into a STAGES-deep
-//                      shared-memory ring.  A P row of the box is one
-//                      128-byte request: the number of row requests an SM
-//                      can have served, not their bytes, bounds how fast it
-//                      streams from HBM (measured on GB300: 64-byte rows
-//                      gave half the bytes per second of 128-byte rows).
+// Roles (11 warps):
+//   warp 0 (one lane)  P producer: per k-block of 128 a 128 x 128 int8 TMA
+//                      box of P (128-byte rows, 128-byte swizzle) into a
+//                      deep ring of its own.  Every row of a TMA box is a
+//                      request of its own; 128-byte rows move twice the
+//                      bytes per request of 64-byte ones (measured on
+//                      GB300: twice the bytes per second per SM).
+//   warp 10 (one lane) Q producer: Q's image with one bulk copy into a
+//                      shallow ring (Q is read from L2).
 //   warps 6..9         converters: lane r of the warp with TMEM lane
 //                      quadrant q converts P row 32 q + r (128 int8, read
 //                      with eight conflict-free 16-byte loads) to 64 packed
@@ -39,12 +42,15 @@
 // Exactness is the general int8 path's: every product is at most 2^14 in
 // magnitude, so a partial sum of at most 1024 of them is an integer below
 // 2^24 in magnitude and exact in fp32; the MMA warp closes the accumulator
-// every 8 k-blocks of 128 (1024 K elements) and the epilogue converts each slab to
-// int32 (exactly) and adds the slabs in int32 registers.
+// every 8 k-blocks of 128 (1024 K elements) and the epilogue converts each
+// slab to int32 (exactly) and adds the slabs in int32 registers.
 //
-// A stage of the ring is free again once the MMAs that read its Q box have
-// completed (tcgen05.commit) and every converter warp has read its P box
-// (one arrival per warp): the empty barrier counts 1 + 4 arrivals.
+// A P stage is free again once every converter warp has read its rows (one
+// arrival per warp), a Q stage once the MMAs that read it have completed
+// (tcgen05.commit), a TMEM P slot likewise.  With P decoupled from the MMA,
+// the P ring keeps its boxes in flight from HBM: measured on GB300, a P box
+// takes about 2 us from issue to arrival under load, so the bytes in flight
+// per SM, not the converters or the MMAs, set the stream rate.
 #include <cuda_bf16.h>
 
 #include "gemm_internal.h"
@@ -55,20 +61,24 @@ namespace {
 
 constexpr int kConvWarps = 4;
 constexpr int kEpiWarps = 4;
-constexpr int kThreadsS8tm = (2 + kEpiWarps + kConvWarps) * 32;  // 320
-constexpr int kKB = kS8tmKB;                                      // K per k-block (stage)
+constexpr int kQWarp = 2 + kEpiWarps + kConvWarps;                // 10: Q producer
+constexpr int kThreadsS8tm = (kQWarp + 1) * 32;                   // 352
+constexpr int kKB = kS8tmKB;                                      // K per k-block
 constexpr uint32_t kPBytes = kBM * kKB;                           // 128 rows x 128 int8
 
-template <int QN, bool Q_KMAJOR, int STAGES, int NA>
+// SP stages of P (16 KB each) and SQ of Q (QN x 256 bytes each) in two
+// separate rings: a P stage is free again as soon as the converters have
+// read it, so the P ring keeps SP boxes in flight from HBM whatever the MMA
+// does; Q comes from L2 and needs only a few stages.
+template <int QN, int SP, int SQ, int NA>
 struct S8tmCfg {
   static_assert(QN == 64 || QN == 128, "QN is 64 or 128");
-  static constexpr uint32_t kQHalf = QN * kRowBytes;  // QN x 64 bf16: one box of Q
-  static constexpr uint32_t kQBytes = 2 * kQHalf;      // the k-block's two halves
-  static constexpr uint32_t kStageBytes = kPBytes + kQBytes;
+  static constexpr uint32_t kQHalf = QN * kRowBytes;  // QN x 64 bf16: one half of a Q image
+  static constexpr uint32_t kQBytes = 2 * kQHalf;      // the k-block's Q image
   static constexpr uint32_t kPOffset = 0;
-  static constexpr uint32_t kQOffset = STAGES * kPBytes;  // 1024-byte aligned
-  static constexpr uint32_t kBarOffset = kQOffset + STAGES * kQBytes;
-  static constexpr uint32_t kNumBars = 2 * STAGES + 2 * NA + 5;
+  static constexpr uint32_t kQOffset = SP * kPBytes;  // 1024-byte aligned
+  static constexpr uint32_t kBarOffset = kQOffset + SQ * kQBytes;
+  static constexpr uint32_t kNumBars = 2 * SP + 2 * SQ + 2 * NA + 5;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
   static constexpr uint32_t kPCol0 = 2 * QN;  // P slots (64 columns each) follow the two accumulators
@@ -120,11 +130,10 @@ __device__ __forceinline__ void store_row(const S8tmParams &p, const int32_t (&a
   }
 }
 
-template <int QN, bool Q_KMAJOR, int STAGES, int NA>
+template <int QN, int SP, int SQ, int NA>
 __global__ void __launch_bounds__(kThreadsS8tm, 1)
-    gemm_s8tm_kernel(const __grid_constant__ CUtensorMap tmP, const __grid_constant__ CUtensorMap tmQ,
-                     const S8tmParams p) {
-  using Cfg = S8tmCfg<QN, Q_KMAJOR, STAGES, NA>;
+    gemm_s8tm_kernel(const __grid_constant__ CUtensorMap tmP, const S8tmParams p) {
+  using Cfg = S8tmCfg<QN, SP, SQ, NA>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-byte alignment
@@ -135,25 +144,32 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(base_ptr + Cfg::kBarOffset + Cfg::kNumBars * 8);
   volatile uint32_t *abort_flag = tmem_slot + 1;
 
-  auto full_bar = [&](uint32_t s) { return bars + 8u * s; };
-  auto empty_bar = [&](uint32_t s) { return bars + 8u * (STAGES + s); };
-  auto pfull_bar = [&](uint32_t a) { return bars + 8u * (2 * STAGES + a); };
-  auto pempty_bar = [&](uint32_t a) { return bars + 8u * (2 * STAGES + NA + a); };
-  auto accf_bar = [&](uint32_t b) { return bars + 8u * (2 * STAGES + 2 * NA + b); };
-  auto acce_bar = [&](uint32_t b) { return bars + 8u * (2 * STAGES + 2 * NA + 2 + b); };
-  const uint32_t drain_bar = bars + 8u * (2 * STAGES + 2 * NA + 4);
+  // P ring, Q ring, TMEM P slots, accumulators
+  auto pfull_bar = [&](uint32_t s) { return bars + 8u * s; };
+  auto pempty_bar = [&](uint32_t s) { return bars + 8u * (SP + s); };
+  auto qfull_bar = [&](uint32_t s) { return bars + 8u * (2 * SP + s); };
+  auto qempty_bar = [&](uint32_t s) { return bars + 8u * (2 * SP + SQ + s); };
+  auto tfull_bar = [&](uint32_t a) { return bars + 8u * (2 * SP + 2 * SQ + a); };
+  auto tempty_bar = [&](uint32_t a) { return bars + 8u * (2 * SP + 2 * SQ + NA + a); };
+  auto accf_bar = [&](uint32_t b) { return bars + 8u * (2 * SP + 2 * SQ + 2 * NA + b); };
+  auto acce_bar = [&](uint32_t b) { return bars + 8u * (2 * SP + 2 * SQ + 2 * NA + 2 + b); };
+  const uint32_t drain_bar = bars + 8u * (2 * SP + 2 * SQ + 2 * NA + 4);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 1 + kConvWarps);
+    for (int s = 0; s < SP; ++s) {
+      mbar_init(pfull_bar(s), 1);
+      mbar_init(pempty_bar(s), kConvWarps);
+    }
+    for (int s = 0; s < SQ; ++s) {
+      mbar_init(qfull_bar(s), 1);
+      mbar_init(qempty_bar(s), 1);
     }
     for (int a = 0; a < NA; ++a) {
-      mbar_init(pfull_bar(a), kConvWarps);
-      mbar_init(pempty_bar(a), 1);
+      mbar_init(tfull_bar(a), kConvWarps);
+      mbar_init(tempty_bar(a), 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(accf_bar(b), 1);
@@ -163,7 +179,6 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
     *abort_flag = 0u;
     fence_mbar_init();
     tma_prefetch_desc(&tmP);
-    tma_prefetch_desc(&tmQ);
   }
   if (warp == 1) tmem_alloc<Cfg::kTmemCols>(smem_addr(tmem_slot));
   tc_fence_before_sync();
@@ -175,44 +190,43 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
   const int num_units = p.tiles_p * p.tiles_q * p.splits;
   constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
 
-  if (warp == 0) {
-    // ------------------------------------------------------ TMA producer
+  if (warp == 0 || warp == kQWarp) {
+    // -------------------------------------------- producers (P, then Q)
     if (lane == 0) {
+      const bool is_p = warp == 0;
+      const int ns = is_p ? SP : SQ;
       uint32_t g = 0;
       bool ok = true;
       for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
         const S8tmUnit w = decode_s8tm(p, u);
         for (int kb = w.kb0; kb < w.kb1; ++kb) {
-          const uint32_t s = g % STAGES, ph = (g / STAGES) & 1u;
-          if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, p.err, p.wait_limit_ns)) {
+          const uint32_t s = g % ns, ph = (g / ns) & 1u;
+          if (!mbar_wait(is_p ? pempty_bar(s) : qempty_bar(s), ph ^ 1u, abort_flag, p.err, p.wait_limit_ns)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(full_bar(s), Cfg::kStageBytes);
-          tma_load_2d(sP + s * kPBytes, &tmP, kb * kKB, w.tp * kBM, full_bar(s));
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const uint32_t q_dst = sQ + s * Cfg::kQBytes + h * Cfg::kQHalf;
-            const int k0 = kb * kKB + h * kBK;
-            if constexpr (Q_KMAJOR) {
-              tma_load_2d(q_dst, &tmQ, k0, w.tq * QN, full_bar(s));
-            } else {
-#pragma unroll
-              for (int j = 0; j < QN / 64; ++j)
-                tma_load_2d(q_dst + j * (kBK * 128), &tmQ, w.tq * QN + 64 * j, k0, full_bar(s));
-            }
+          if (is_p) {
+            mbar_arrive_expect_tx(pfull_bar(s), kPBytes);
+            tma_load_2d(sP + s * kPBytes, &tmP, kb * kKB, w.tp * kBM, pfull_bar(s));
+          } else {
+            mbar_arrive_expect_tx(qfull_bar(s), Cfg::kQBytes);
+            const uint8_t *q_src = static_cast<const uint8_t *>(p.q_img) +
+                                   ((int64_t)w.tq * p.num_kb + kb) * (int64_t)Cfg::kQBytes;
+            bulk_load(sQ + s * Cfg::kQBytes, q_src, Cfg::kQBytes, qfull_bar(s));
           }
           ++g;
         }
       }
-      const uint32_t first = g > (uint32_t)STAGES ? g - STAGES : 0u;
-      for (uint32_t i = first; i < g; ++i) mbar_wait_drain(full_bar(i % STAGES), (i / STAGES) & 1u, kDrainNs);
+      // Every copy this thread issued has landed before the CTA may exit.
+      const uint32_t first = g > (uint32_t)ns ? g - ns : 0u;
+      for (uint32_t i = first; i < g; ++i)
+        mbar_wait_drain(is_p ? pfull_bar(i % ns) : qfull_bar(i % ns), (i / ns) & 1u, kDrainNs);
     }
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kBM, QN, !Q_KMAJOR);
+      constexpr uint32_t idesc = idesc_bf16_f32(kBM, QN, false);
       uint32_t g = 0, acc_cnt = 0;
       bool ok = true;
       for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
@@ -227,10 +241,10 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
           tc_fence_after_sync();
           const uint32_t d_tmem = tmem_base + b * QN;
           for (int kb = kb_s; kb < kb_e; ++kb) {
-            const uint32_t s = g % STAGES, ph = (g / STAGES) & 1u;
-            const uint32_t a = g % NA, pph = (g / NA) & 1u;
-            if (!mbar_wait(full_bar(s), ph, abort_flag, p.err, p.wait_limit_ns) ||
-                !mbar_wait(pfull_bar(a), pph, abort_flag, p.err, p.wait_limit_ns)) {
+            const uint32_t s = g % SQ, ph = (g / SQ) & 1u;
+            const uint32_t a = g % NA, tph = (g / NA) & 1u;
+            if (!mbar_wait(qfull_bar(s), ph, abort_flag, p.err, p.wait_limit_ns) ||
+                !mbar_wait(tfull_bar(a), tph, abort_flag, p.err, p.wait_limit_ns)) {
               ok = false;
               break;
             }
@@ -239,17 +253,15 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
             const uint32_t a_tmem = tmem_base + Cfg::kPCol0 + a * 64;
 #pragma unroll
             for (int k = 0; k < kKB / 16; ++k) {
-              // one K step of 16 is 8 packed columns of the P slot; Q as B
-              // in the general kernel, within the half k / 4 (K-major: 32
-              // bytes along a row; MN-major: 16 K rows = 2048 bytes, 64-wide
-              // chunks 8 KB apart)
+              // one K step of 16 is 8 packed columns of the P slot, and 32
+              // bytes along the rows of Q's half k / 4 (K-major, 128-byte
+              // swizzle, 8-row atoms 1024 bytes apart)
               const uint32_t qh = q0 + (k >> 2) * Cfg::kQHalf, kk = k & 3;
-              const uint64_t bd = Q_KMAJOR ? smem_desc_sw128(qh + kk * 32, 16, 1024)
-                                           : smem_desc_sw128(qh + kk * 2048, kBK * 128, 1024);
+              const uint64_t bd = smem_desc_sw128(qh + kk * 32, 16, 1024);
               tc_mma_bf16_tmem_a(d_tmem, a_tmem + k * 8, bd, idesc, (kb > kb_s || k > 0) ? 1u : 0u);
             }
-            tc_commit(empty_bar(s));   // the Q box may be overwritten once these MMAs finish
-            tc_commit(pempty_bar(a));  // and the P slot reused
+            tc_commit(qempty_bar(s));  // the Q stage may be refilled once these MMAs finish
+            tc_commit(tempty_bar(a));  // and the P slot reused
             ++g;
           }
           if (!ok) break;
@@ -278,16 +290,16 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
       tmem_st_wait();
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(pfull_bar(slot));
+      if (lane == 0) mbar_arrive(tfull_bar(slot));
       __syncwarp();
     };
     for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
       const S8tmUnit w = decode_s8tm(p, u);
       for (int kb = w.kb0; kb < w.kb1; ++kb) {
-        const uint32_t s = g % STAGES, ph = (g / STAGES) & 1u;
-        const uint32_t a = g % NA, pph = (g / NA) & 1u;
-        if (!__all_sync(0xffffffffu, mbar_wait(full_bar(s), ph, abort_flag, p.err, p.wait_limit_ns)) ||
-            !__all_sync(0xffffffffu, mbar_wait(pempty_bar(a), pph ^ 1u, abort_flag, p.err, p.wait_limit_ns))) {
+        const uint32_t s = g % SP, ph = (g / SP) & 1u;
+        const uint32_t a = g % NA, tph = (g / NA) & 1u;
+        if (!__all_sync(0xffffffffu, mbar_wait(pfull_bar(s), ph, abort_flag, p.err, p.wait_limit_ns)) ||
+            !__all_sync(0xffffffffu, mbar_wait(tempty_bar(a), tph ^ 1u, abort_flag, p.err, p.wait_limit_ns))) {
           ok = false;
           break;
         }
@@ -303,7 +315,7 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
           s8x4_to_bf16x4(v.w, o[8 * j + 6], o[8 * j + 7]);
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(empty_bar(s));  // this warp's rows of the P box are read
+        if (lane == 0) mbar_arrive(pempty_bar(s));  // this warp's rows of the P box are read
         __syncwarp();
         if (pending) publish(pending_slot);
         tmem_st_32x32b_x64(lane_base + a * 64, o);
@@ -368,24 +380,73 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
   }
 }
 
-template <int QN, bool Q_KMAJOR, int STAGES, int NA>
-cudaError_t launch_one(const CUtensorMap &tp, const CUtensorMap &tq, const S8tmParams &p, int grid,
-                       cudaStream_t st) {
-  using Cfg = S8tmCfg<QN, Q_KMAJOR, STAGES, NA>;
-  auto kern = gemm_s8tm_kernel<QN, Q_KMAJOR, STAGES, NA>;
+// Q's image for one (Q tile, k-block): QN rows x 128 K of bf16 as two
+// 64-K halves of QN 128-byte rows, 16-byte chunk j of row r stored at chunk
+// j ^ (r % 8) (the 128-byte swizzle).  One thread writes one 16-byte chunk
+// (8 consecutive k of one row), reading Q(q, k) at src + q * sq + k * sk.
+__global__ void __launch_bounds__(256)
+    s8tm_stage_q_kernel(const int8_t *__restrict__ src, int64_t sq, int64_t sk, int Q_rows, int K, int qn,
+                        int num_kb, uint4 *__restrict__ img, int64_t chunks) {
+  griddep_launch_dependents();  // the GEMM waits for completion before reading
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= chunks) return;
+  const int per_tile = 2 * qn * 8;  // 16-byte chunks per image
+  const int64_t tile = t / per_tile;
+  const int c = (int)(t - tile * per_tile);
+  const int h = c / (qn * 8), rem = c - h * (qn * 8);
+  const int row = rem >> 3, j = rem & 7;
+  const int64_t tq = tile / num_kb, kb = tile - tq * num_kb;
+  const int64_t q = tq * qn + row, k0 = kb * kKB + h * 64 + j * 8;
+  uint32_t w[2] = {0u, 0u};
+  if (q < Q_rows) {
+    const int8_t *s = src + q * sq + k0 * sk;
+    if (sk == 1 && k0 + 8 <= K && (reinterpret_cast<uintptr_t>(s) & 7) == 0) {
+      const uint2 v = *reinterpret_cast<const uint2 *>(s);
+      w[0] = v.x;
+      w[1] = v.y;
+    } else {
+      for (int i = 0; i < 8; ++i)
+        if (k0 + i < K) w[i >> 2] |= (uint32_t)(uint8_t)s[i * sk] << (8 * (i & 3));
+    }
+  }
+  uint4 o;
+  s8x4_to_bf16x4(w[0], o.x, o.y);
+  s8x4_to_bf16x4(w[1], o.z, o.w);
+  const int64_t at = tile * per_tile + h * (qn * 8) + row * 8 + (j ^ (row & 7));
+  img[at] = o;
+}
+
+template <int QN, int SP, int SQ, int NA>
+cudaError_t launch_one(const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st) {
+  using Cfg = S8tmCfg<QN, SP, SQ, NA>;
+  auto kern = gemm_s8tm_kernel<QN, SP, SQ, NA>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmemBytes);
   if (e != cudaSuccess) return e;
-  return launch_ex(kern, dim3(grid), dim3(kThreadsS8tm), Cfg::kSmemBytes, st, 1, tp, tq, p);
+  return launch_ex(kern, dim3(grid), dim3(kThreadsS8tm), Cfg::kSmemBytes, st, 1, tp, p);
 }
 
 }  // namespace
 
-cudaError_t launch_s8tm(int qn, bool q_kmajor, const CUtensorMap &tp, const CUtensorMap &tq, const S8tmParams &p,
-                        int grid, cudaStream_t st) {
-  // stages: 4 x 48 KB (QN 128) or 6 x 32 KB (QN 64) of operands in flight
-  if (qn == 128)
-    return q_kmajor ? launch_one<128, true, 4, 4>(tp, tq, p, grid, st) : launch_one<128, false, 4, 4>(tp, tq, p, grid, st);
-  return q_kmajor ? launch_one<64, true, 6, 4>(tp, tq, p, grid, st) : launch_one<64, false, 6, 4>(tp, tq, p, grid, st);
+size_t s8tm_q_image_bytes(int qn, int64_t Q_rows, int64_t K) {
+  const int64_t tiles_q = (Q_rows + qn - 1) / qn, num_kb = (K + kKB - 1) / kKB;
+  return (size_t)tiles_q * num_kb * 2 * qn * 128;
+}
+
+cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64_t Q_rows, int64_t K, int qn,
+                                void *img, cudaStream_t st) {
+  const int64_t num_kb = (K + kKB - 1) / kKB;
+  const int64_t chunks = (int64_t)s8tm_q_image_bytes(qn, Q_rows, K) / 16;
+  if (chunks == 0) return cudaSuccess;
+  s8tm_stage_q_kernel<<<(unsigned)((chunks + 255) / 256), 256, 0, st>>>(src, sq, sk, (int)Q_rows, (int)K, qn,
+                                                                       (int)num_kb, static_cast<uint4 *>(img), chunks);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_s8tm(int qn, const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st) {
+  // P stages x 16 KB + Q stages x (QN x 256 bytes): 9 x 16 + 2 x 32 KB
+  // (QN 128) or 10 x 16 + 3 x 16 KB (QN 64)
+  if (qn == 128) return launch_one<128, 9, 2, 4>(tp, p, grid, st);
+  return launch_one<64, 10, 3, 4>(tp, p, grid, st);
 }
 
 }  // namespace gb300
