@@ -411,11 +411,12 @@ def run_ours(args, rank, world, dev):
 
 
 def kernel_source_hash() -> str:
-    """Hash of the tensor-core kernel's sources: counters taken from an older
-    kernel are not reported as this kernel's."""
+    """Hash of the main kernels' sources (tensor-core kernels, the int8
+    kernel that converts in tensor memory, the small-M kernel): counters
+    taken from an older kernel are not reported as this kernel's."""
     import hashlib
     h = hashlib.sha256()
-    for f in ("gemm_tc.cuh", "gemm_tc2.cuh", "ptx.cuh"):
+    for f in ("gemm_tc.cuh", "gemm_tc2.cuh", "ptx.cuh", "gemm_s8tm.cu", "gemm_skinny.cu"):
         with open(os.path.join(ROOT, "paper_2512_13282_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
