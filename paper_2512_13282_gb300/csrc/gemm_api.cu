@@ -114,7 +114,8 @@ gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
 // GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
 // split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
 // CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores, GB300_GEMM_PDL=0
-// plain stream ordering; GB300_GEMM_DEBUG=1 (read once) prints each plan.
+// plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
+// small-operand shapes; GB300_GEMM_DEBUG=1 (read once) prints each plan.
 int env_int(const char *name) {
   const char *s = std::getenv(name);
   return s ? std::atoi(s) : 0;
