@@ -560,8 +560,11 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   const int64_t kb_per = ceil_div(num_kb, splits);
   splits = ceil_div(num_kb, kb_per);
   gemm_status_t s;
+  // split-K: int32 outputs are added into C (zeroed by the staging launch),
+  // int16 / int8 ones go through int32 partials and the reduction kernel
+  const bool add_into_c = splits > 1 && out_bits == 32;
   const size_t q_bytes = align_up(s8tm_q_image_bytes(qn, Q_rows, K), 256);
-  const size_t total = q_bytes + (splits > 1 ? (size_t)splits * M * N * 4 : 0);
+  const size_t total = q_bytes + (splits > 1 && !add_into_c ? (size_t)splits * M * N * 4 : 0);
   if ((s = ensure_workspace(d, total, st)) != GEMM_OK) {
     *status = s;
     return true;
@@ -569,7 +572,9 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   uint8_t *ws = static_cast<uint8_t *>(d.ws);
   *status = GEMM_ERR_CUDA;
   g_launches.fetch_add(1);
-  if (launch_s8tm_stage_q(Qs, sq, sk, Q_rows, K, qn, ws, st) != cudaSuccess) return true;
+  if (launch_s8tm_stage_q(Qs, sq, sk, Q_rows, K, qn, ws, add_into_c ? static_cast<int32_t *>(C) : nullptr, M, N,
+                          ldc, st) != cudaSuccess)
+    return true;
   CUtensorMap tp;
   if (!encode_s8_rows(&tp, P, (uint64_t)K, (uint64_t)P_rows, (uint64_t)ldp)) return true;
   S8tmParams p{};
@@ -587,7 +592,7 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   p.swap = swap ? 1 : 0;
   p.C = C;
   p.ldc = ldc;
-  p.ws = splits > 1 ? ws + q_bytes : nullptr;
+  p.ws = splits > 1 && !add_into_c ? ws + q_bytes : nullptr;
   p.err = d.err;
   p.wait_limit_ns = wait_limit_ns();
   p.out_bits = out_bits;
@@ -605,7 +610,7 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   g_launches.fetch_add(1);
   if (launch_s8tm(qn, tp, p, grid, st) != cudaSuccess) return true;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
-  if (splits > 1) {
+  if (splits > 1 && !add_into_c) {
     g_launches.fetch_add(1);
     if (launch_splitk_reduce_s32(static_cast<const int32_t *>(p.ws), (int)splits, M, N, C, ldc, out_bits, shift,
                                  d.sms, st) != cudaSuccess)

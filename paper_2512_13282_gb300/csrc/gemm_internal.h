@@ -89,7 +89,8 @@ struct S8tmParams {
   int swap;
   void *C;
   int64_t ldc;
-  void *ws;          // split-K partials: splits x M x N int32 (row pitch N)
+  void *ws;          // split-K partials of int16 / int8 outputs: splits x M x N int32 (row pitch N);
+                     // int32 outputs with split-K are added into C, zeroed beforehand
   uint32_t *err;
   uint64_t wait_limit_ns;
   int out_bits;      // 32, 16 or 8
@@ -98,9 +99,12 @@ struct S8tmParams {
 };
 // Bytes of Q's images for QN = qn columns per tile.
 size_t s8tm_q_image_bytes(int qn, int64_t Q_rows, int64_t K);
-// Writes Q's images: Q(q, k) = src[q * sq + k * sk] (int8), exact bf16.
+// Writes Q's images: Q(q, k) = src[q * sq + k * sk] (int8), exact bf16;
+// when zero_c is not null, also sets the c_rows x c_cols int32 matrix at
+// zero_c (row pitch ldc) to zero.
 cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64_t Q_rows, int64_t K, int qn,
-                                void *img, cudaStream_t st);
+                                void *img, int32_t *zero_c, int64_t c_rows, int64_t c_cols, int64_t ldc,
+                                cudaStream_t st);
 // qn: 64 or 128 columns of Q per tile.
 cudaError_t launch_s8tm(int qn, const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st);
 

@@ -111,7 +111,14 @@ template <int QN>
 __device__ __forceinline__ void store_row(const S8tmParams &p, const int32_t (&acc)[QN], int split, int64_t off0,
                                           int64_t step, int64_t q0) {
   const int64_t nq = p.Q_rows - q0;  // valid elements (>= 1)
-  if (p.splits > 1 || p.out_bits == 32) {
+  if (p.splits > 1 && p.out_bits == 32) {
+    // int32 C, zeroed by the Q staging kernel: every split adds its exact
+    // partial sums (integer addition, so any order gives the same C)
+    int32_t *dst = reinterpret_cast<int32_t *>(p.C) + off0;
+#pragma unroll
+    for (int i = 0; i < QN; ++i)
+      if (i < nq) atomicAdd(dst + i * step, acc[i]);
+  } else if (p.splits > 1 || p.out_bits == 32) {
     int32_t *dst = reinterpret_cast<int32_t *>(p.splits > 1 ? p.ws : p.C) +
                    (p.splits > 1 ? (int64_t)split * p.M * p.N : 0) + off0;
 #pragma unroll
@@ -360,8 +367,8 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
       const int64_t prow = (int64_t)w.tp * kBM + r;
       if (prow >= p.P_rows) continue;
       const int64_t q0 = (int64_t)w.tq * QN;
-      // partials have row pitch N; C has ldc
-      const int64_t ld = p.splits > 1 ? (int64_t)p.N : p.ldc;
+      // partials (split-K of int16 / int8 outputs) have row pitch N; C has ldc
+      const int64_t ld = (p.splits > 1 && p.out_bits != 32) ? (int64_t)p.N : p.ldc;
       if (p.swap)  // C[q][prow]: per element the warp's lanes store 32 consecutive columns
         store_row<QN>(p, acc, w.split, q0 * ld + prow, ld, q0);
       else         // C[prow][q]
@@ -386,10 +393,18 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
 // (8 consecutive k of one row), reading Q(q, k) at src + q * sq + k * sk.
 __global__ void __launch_bounds__(256)
     s8tm_stage_q_kernel(const int8_t *__restrict__ src, int64_t sq, int64_t sk, int Q_rows, int K, int qn,
-                        int num_kb, uint4 *__restrict__ img, int64_t chunks) {
+                        int num_kb, uint4 *__restrict__ img, int64_t chunks, int32_t *__restrict__ zero_c,
+                        int64_t c_rows, int64_t c_cols, int64_t ldc) {
   griddep_launch_dependents();  // the GEMM waits for completion before reading
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= chunks) return;
+  if (t >= chunks) {  // the remaining threads zero C (int32, split-K by atomic adds)
+    const int64_t total = c_rows * c_cols;
+    for (int64_t e = t - chunks; zero_c && e < total; e += (int64_t)gridDim.x * blockDim.x - chunks) {
+      const int64_t r = e / c_cols;
+      zero_c[r * ldc + (e - r * c_cols)] = 0;
+    }
+    return;
+  }
   const int per_tile = 2 * qn * 8;  // 16-byte chunks per image
   const int64_t tile = t / per_tile;
   const int c = (int)(t - tile * per_tile);
@@ -433,12 +448,16 @@ size_t s8tm_q_image_bytes(int qn, int64_t Q_rows, int64_t K) {
 }
 
 cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64_t Q_rows, int64_t K, int qn,
-                                void *img, cudaStream_t st) {
+                                void *img, int32_t *zero_c, int64_t c_rows, int64_t c_cols, int64_t ldc,
+                                cudaStream_t st) {
   const int64_t num_kb = (K + kKB - 1) / kKB;
   const int64_t chunks = (int64_t)s8tm_q_image_bytes(qn, Q_rows, K) / 16;
-  if (chunks == 0) return cudaSuccess;
-  s8tm_stage_q_kernel<<<(unsigned)((chunks + 255) / 256), 256, 0, st>>>(src, sq, sk, (int)Q_rows, (int)K, qn,
-                                                                       (int)num_kb, static_cast<uint4 *>(img), chunks);
+  // 64K more threads zero C when asked (a grid-stride loop over its elements)
+  const int64_t extra = zero_c ? 65536 : 0;
+  if (chunks + extra == 0) return cudaSuccess;
+  s8tm_stage_q_kernel<<<(unsigned)((chunks + extra + 255) / 256), 256, 0, st>>>(
+      src, sq, sk, (int)Q_rows, (int)K, qn, (int)num_kb, static_cast<uint4 *>(img), chunks, zero_c, c_rows, c_cols,
+      ldc);
   return cudaGetLastError();
 }
 

@@ -398,3 +398,16 @@ def test_int8_converted_in_kernel_matches_general_path(M, N, K, layout, monkeypa
     assert np.array_equal(C0, C1)
     r, c = _sample_positions(M, N, seed=3)
     assert np.array_equal(C1[r, c].astype(np.int64), oracle.gemm_s8_entries(A, B, layout, r, c))
+
+
+@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (100, 1000, 3000, COL), (1000, 64, 3008, ROW)],
+                         ids=["swap", "swap-ragged", "direct"])
+@pytest.mark.parametrize("splits", ["3", "8"])
+def test_int8_converted_in_kernel_split_into_padded_c(M, N, K, layout, splits, monkeypatch):
+    """Split-K of int32 outputs on the small-operand path adds every split's
+    exact partial sums into C, zeroed beforehand: C with a padded pitch and
+    an offset base, nothing outside [0,M) x [0,N) written."""
+    monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
+    A, B = _inputs("int8", M, N, K, layout, seed=M + K)
+    C = U.run("int8", A, B, layout, ldc=N + 5, c_off=3)
+    _check("int8", A, B, layout, C)
