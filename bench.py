@@ -410,13 +410,21 @@ def run_ours(args, rank, world, dev):
     return line
 
 
-def kernel_source_hash() -> str:
-    """Hash of the main kernels' sources (tensor-core kernels, the int8
-    kernel that converts in tensor memory, the small-M kernel): counters
-    taken from an older kernel are not reported as this kernel's."""
+# Source files that determine each kernel family's code: DRAM counters of a
+# family are reported only while these files hash to the recorded value.
+KERNEL_FAMILIES = {
+    "tc": ("gemm_tc.cuh", "gemm_tc2.cuh", "ptx.cuh"),
+    "s8tm": ("gemm_s8tm.cu", "ptx.cuh"),
+    "skinny": ("gemm_skinny.cu", "ptx.cuh"),
+}
+
+
+def kernel_source_hash(family: str = "tc") -> str:
+    """Hash of one kernel family's sources: counters taken from an older
+    kernel are not reported as this kernel's."""
     import hashlib
     h = hashlib.sha256()
-    for f in ("gemm_tc.cuh", "gemm_tc2.cuh", "ptx.cuh", "gemm_s8tm.cu", "gemm_skinny.cu"):
+    for f in KERNEL_FAMILIES[family]:
         with open(os.path.join(ROOT, "paper_2512_13282_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -453,14 +461,15 @@ def bound_of(g: W.Gemm, tflops_peak: float, gbs_peak: float) -> str:
 def load_traffic(name):
     """DRAM bytes (read + write) per launch of the dominant kernel from the
     committed ncu summary (profiles/traffic.json), or None when it was not
-    captured for this GEMM or the kernel source has changed since."""
+    captured for this GEMM or its kernel family's source has changed since."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(p) as f:
             d = json.load(f)
-        if d.get("kernel_source_hash") != kernel_source_hash():
+        e = d.get("dram_bytes_per_launch", {}).get(name)
+        if not e or d.get("kernel_source_hash", {}).get(e["family"]) != kernel_source_hash(e["family"]):
             return None
-        return d.get("dram_bytes_per_launch", {}).get(name)
+        return e["bytes"]
     except Exception:
         return None
 
