@@ -192,7 +192,12 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
-  griddep_wait();  // the staged Q comes from the previous kernel of the stream
+  // The previous kernel of the stream is the Q staging launch (a plain
+  // launch: everything before it on the stream completed before it began).
+  // It writes Q's images and, for split-K into int32 C, zeroes C: the Q
+  // producer and the epilogue wait for it (griddep_wait) before touching
+  // those, while P, written before the staging launch began, is streamed at
+  // once, so that the P ring fills while the staging kernel still runs.
 
   const int num_units = p.tiles_p * p.tiles_q * p.splits;
   constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
@@ -201,6 +206,7 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
     // -------------------------------------------- producers (P, then Q)
     if (lane == 0) {
       const bool is_p = warp == 0;
+      if (!is_p) griddep_wait();
       const int ns = is_p ? SP : SQ;
       uint32_t g = 0;
       bool ok = true;
@@ -334,6 +340,7 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
     if (pending) publish(pending_slot);
   } else {
     // --------------------------------------------------------- epilogue
+    griddep_wait();  // C (zeroed by the staging launch) is written below
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
     uint32_t acc_cnt = 0;
