@@ -32,10 +32,12 @@
  *     benchmarks (int8 results are identical either way; bf16 results may
  *     differ in summation order, within the same accuracy): GB300_GEMM_BN,
  *     GB300_GEMM_PAIR, GB300_GEMM_SPLITS, GB300_GEMM_SKINNY_MAX_M,
- *     GB300_GEMM_TMA_STORE=0, GB300_GEMM_PDL=0 and GB300_GEMM_S8TM=0 (int8
+ *     GB300_GEMM_TMA_STORE=0, GB300_GEMM_PDL=0, GB300_GEMM_S8TM=0 (int8
  *     GEMMs with one operand of at most 128 rows take the general path
- *     instead of converting the large operand inside the kernel), read at
- *     every call.
+ *     instead of converting the large operand inside the kernel) and
+ *     GB300_GEMM_S8A=1 (int8 GEMMs planned as 128 x 224 tiles convert A
+ *     inside the kernel instead of staging it; slower, off by default), read
+ *     at every call.
  *     GB300_GEMM_WAIT_LIMIT_MS (read once) bounds every device-side wait
  *     (default 2000 ms); GB300_GEMM_DEBUG=1 prints each plan to stderr.
  */

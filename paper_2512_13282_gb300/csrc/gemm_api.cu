@@ -115,7 +115,9 @@ gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
 // split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
 // CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores, GB300_GEMM_PDL=0
 // plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
-// small-operand shapes; GB300_GEMM_DEBUG=1 (read once) prints each plan.
+// small-operand shapes, GB300_GEMM_S8A=1 the int8 kernel that converts A in
+// tensor memory for 224-wide tiles; GB300_GEMM_DEBUG=1 (read once) prints
+// each plan.
 int env_int(const char *name) {
   const char *s = std::getenv(name);
   return s ? std::atoi(s) : 0;
@@ -620,6 +622,71 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   return true;
 }
 
+// int8 A of gemm_s8a_kernel: boxes of 64 bytes x 128 rows, 64-byte swizzle.
+bool encode_s8_rows64(CUtensorMap *map, const void *base, uint64_t K, uint64_t rows, uint64_t ld) {
+  const cuuint64_t dims[2] = {K, rows};
+  const cuuint64_t strides[1] = {ld};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kBM};
+  const cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Compute-bound int8 GEMMs planned as single-CTA 128 x 224 tiles without
+// split-K, with A TMA-legal as int8 (16-byte aligned base and pitch):
+// gemm_s8a_kernel converts A in the kernel, so only B is staged.  Off unless
+// GB300_GEMM_S8A=1: exact, but measured slower than staging both operands
+// (int8 4096^3: 151 against 110 us).  Returns false, having launched
+// nothing, when it is off or the plan or A rules it out.
+bool try_s8a(DeviceState &d, Plan &pl, const int8_t *A, int64_t lda, const int8_t *B, int64_t ldb, bool b_kmajor,
+             void *C, int64_t ldc, int out_esize, cudaStream_t st, gemm_status_t *status) {
+  const char *env = std::getenv("GB300_GEMM_S8A");
+  if (!env || std::atoi(env) != 1) return false;
+  TcParams &p = pl.p;
+  if (pl.v.pair || pl.v.bn != 224 || !b_kmajor || p.splits != 1 || !aligned16(A) || lda % 16 != 0) return false;
+  const int64_t N = p.N, K = p.K;
+  const int64_t ldb_p = (K + 7) / 8 * 8;  // B stored N x K, staged with 16-byte aligned rows
+  gemm_status_t s;
+  if ((s = ensure_workspace(d, align_up((size_t)N * ldb_p * 2, 256), st)) != GEMM_OK) {
+    *status = s;
+    return true;
+  }
+  uint16_t *Bb = static_cast<uint16_t *>(d.ws);
+  *status = GEMM_ERR_CUDA;
+  g_launches.fetch_add(1);
+  if (launch_s8_to_bf16_pair(S8Job{B, N, K, ldb, Bb, ldb_p}, S8Job{nullptr, 0, 0, 0, nullptr, 0}, d.sms, st) !=
+      cudaSuccess)
+    return true;
+  CUtensorMap ta, tb, tout;
+  if (!encode_s8_rows64(&ta, A, (uint64_t)K, (uint64_t)p.M, (uint64_t)lda)) return true;
+  if (!encode_bf16_2d(&tb, Bb, (uint64_t)K, (uint64_t)N, (uint64_t)ldb_p, kBK, 224)) return true;
+  p.C = C;
+  p.ldc = ldc;
+  p.c_vec = aligned16(C) && ((ldc * out_esize) % 16 == 0);
+  p.ws = nullptr;
+  p.out_tma = kOutDirect;
+  tout = ta;
+  const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
+  if (p.c_vec && !(tma_env && std::atoi(tma_env) == 0)) {
+    const CUtensorMapDataType type = p.out_bits == 32   ? CU_TENSOR_MAP_DATA_TYPE_INT32
+                                     : p.out_bits == 16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16
+                                                        : CU_TENSOR_MAP_DATA_TYPE_UINT8;
+    if (!encode_out(&tout, type, (uint32_t)out_esize, C, (uint64_t)N, (uint64_t)p.M, (uint64_t)ldc, 1, 32))
+      return true;
+    p.out_tma = kOutTmaC;
+  }
+  p.err = d.err;
+  p.wait_limit_ns = wait_limit_ns();
+  const bool prof = g_prof_start && g_prof_stop;
+  if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
+  g_launches.fetch_add(1);
+  if (launch_s8a(ta, tb, tout, p, pl.grid, st) != cudaSuccess) return true;
+  if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
+  *status = GEMM_OK;
+  return true;
+}
+
 // The int8 GEMM behind gemm_s8s8_s32 (out_bits 32), gemm_s8s8_s16 and
 // gemm_s8s8_s8 (out_bits 16 / 8, right shift `shift`): the exact int32 sum
 // is formed the same way for all three; only the final store differs.
@@ -646,6 +713,7 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
   pl.p.out_bits = out_bits;
   pl.p.out_shift = shift;
+  if (try_s8a(*d, pl, A, lda, B, ldb, b_kmajor, C, ldc, out_esize, st, &s)) return s;
   // Stage both operands as bf16 (exact for int8) with 16-byte aligned rows.
   const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
   const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;

@@ -108,6 +108,12 @@ cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64
 // qn: 64 or 128 columns of Q per tile.
 cudaError_t launch_s8tm(int qn, const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st);
 
+// int8 GEMM with single-CTA 128 x 224 tiles, A (int8, TMA boxes of 64 x 128)
+// converted in the kernel into TMEM and B staged as bf16, stored N x K
+// (gemm_s8a.cu); p.splits must be 1.
+cudaError_t launch_s8a(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p, int grid,
+                       cudaStream_t st);
+
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
 // int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is
 // rows x cols with an arbitrary source leading dimension.

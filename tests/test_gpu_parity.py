@@ -411,3 +411,27 @@ def test_int8_converted_in_kernel_split_into_padded_c(M, N, K, layout, splits, m
     A, B = _inputs("int8", M, N, K, layout, seed=M + K)
     C = U.run("int8", A, B, layout, ldc=N + 5, c_off=3)
     _check("int8", A, B, layout, C)
+
+
+# ---------------- int8 compute-bound tiles with A converted in tensor memory
+
+@pytest.mark.parametrize("M,N,K", [(300, 700, 1504), (130, 450, 3008), (1000, 2000, 4096), (2048, 4096, 1024)],
+                         ids=["ragged", "two-slab-tail", "mid", "wide"])
+@pytest.mark.parametrize("out", ["int8", "int8_int16"])
+def test_int8_a_converted_in_kernel(M, N, K, out, monkeypatch):
+    """Single-CTA 128 x 224 tiles without split-K and an aligned A, with the
+    kernel that converts A in TMEM turned on (GB300_GEMM_S8A=1; it is off by
+    default): A is streamed as int8, only B is staged.  Bit-exact against the
+    oracle and equal to the staged path."""
+    monkeypatch.setenv("GB300_GEMM_BN", "224")
+    monkeypatch.setenv("GB300_GEMM_PAIR", "0")
+    monkeypatch.setenv("GB300_GEMM_SPLITS", "1")
+    monkeypatch.setenv("GB300_GEMM_S8A", "1")
+    A, B = _inputs("int8", M, N, K, COL, seed=M + N)
+    C = U.run(out, A, B, COL, shift=7)
+    if out == "int8":
+        _check("int8", A, B, COL, C)
+    else:
+        assert np.array_equal(C.astype(np.int64), oracle.requantize(oracle.gemm_s8(A, B, COL), 7, 16))
+    monkeypatch.setenv("GB300_GEMM_S8A", "0")
+    assert np.array_equal(U.run(out, A, B, COL, shift=7), C)
