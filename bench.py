@@ -351,11 +351,7 @@ def run_ours(args, rank, world, dev):
             if not ok:
                 raise RuntimeError(f"{c.g.name}: host-buffer results differ from the whole-matrix call")
 
-    # max over ranks
-    vals = torch.tensor([gemm_ms, e2e_ms or 0.0, wall], dtype=torch.float64, device=dev)
-    if world > 1:
-        torch.distributed.all_reduce(vals, op=torch.distributed.ReduceOp.MAX)
-    gemm_ms, e2e_max, wall = vals.tolist()
+    gemm_ms, e2e_max, wall = max_over_ranks([gemm_ms, e2e_ms or 0.0, wall], world, dev)
 
     peaks, peak_src = load_peaks()
     bf16_peak = float(peaks.get("bf16_tflops", FALLBACK["bf16_tflops"]))
@@ -388,7 +384,7 @@ def run_ours(args, rank, world, dev):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(wl, args.cpu_seconds)
 
-    value = world * ops / (gemm_ms * 1e-3) / 1e12
+    value = whole_job_tops(ops, world, gemm_ms)
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(gemm_ms, 5),
@@ -400,7 +396,7 @@ def run_ours(args, rank, world, dev):
         "per_gemm": per,
         "roofline": roof,
         "e2e": None if e2e_ms is None else {
-            "value": round(world * ops / (e2e_max * 1e-3) / 1e12, 3), "unit": "TOPS",
+            "value": round(whole_job_tops(ops, world, e2e_max), 3), "unit": "TOPS",
             "h2d_bytes_per_step": sum(c.h2d for c in cases), "d2h_bytes_per_step": sum(c.d2h for c in cases)},
         "gpu_launches": int(launches),
         "wall_s_timed_region": round(wall, 4),
@@ -417,6 +413,22 @@ KERNEL_FAMILIES = {
     "s8tm": ("gemm_s8tm.cu", "ptx.cuh"),
     "skinny": ("gemm_skinny.cu", "ptx.cuh"),
 }
+
+
+def max_over_ranks(values, world, device):
+    """Element-wise maximum of per-rank timings over all ranks (a job of
+    replicas takes as long as its slowest rank); the values unchanged on one
+    rank."""
+    vals = torch.tensor(values, dtype=torch.float64, device=device)
+    if world > 1:
+        torch.distributed.all_reduce(vals, op=torch.distributed.ReduceOp.MAX)
+    return vals.tolist()
+
+
+def whole_job_tops(ops_per_rank, world, ms):
+    """Throughput of `world` replicas that each do ops_per_rank operations,
+    over the slowest rank's time `ms` (milliseconds), in TOPS."""
+    return world * ops_per_rank / (ms * 1e-3) / 1e12
 
 
 def kernel_source_hash(family: str = "tc") -> str:
