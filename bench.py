@@ -1,11 +1,19 @@
 """Benchmark of the GB300 dense GEMM library (C = A.B, int8->int32 exact and
 bf16->fp32->bf16 RNE).
 
-One step = every GEMM of the chosen workload once (default: the square sweep
-M=N=K in {512,1024,2048,4096}, int8 and bf16, B column-major).  Inputs are
-seeded synthetic matrices (workloads.py) resident in HBM before timing.  L2
-(129 MB) is flushed by writing a 512 MiB buffer before every timed GEMM; each
-GEMM is bracketed by CUDA events on its stream, so flushes are not timed.
+One step = every GEMM of the chosen workload once (default: all 37 GEMMs of
+the five benchmark configurations -- int8 256^3, the square sweep
+512..4096 of both paths, 8192^3 of both paths, the transformer projections
+and the irregular/skinny shapes).  Inputs are seeded synthetic matrices
+(workloads.py) resident in HBM before timing.  L2 (129 MB) is flushed by
+writing a 512 MiB buffer before every timed GEMM; each GEMM is bracketed by
+CUDA events on its stream, so flushes are not timed.  The flush leaves dirty
+lines in L2 whose write-back lands in the next GEMM, so a second pass times
+every GEMM again after a clean flush (the same write, then a 256 MiB read of
+another buffer) and reports both per GEMM.  For HBM-bound GEMMs, the time of
+a plain read of the same compulsory bytes after the same flush (the
+library's read-bandwidth diagnostic: 16-byte loads, nothing kept) is measured
+beside it: the ceiling an isolated call of that size can reach.
 
   value       whole-job throughput, sum(2*M*N*K) / sum(event time), in TOPS
               (tera-ops/s; int8 MACs and bf16 FMAs both count 2 ops)
@@ -52,6 +60,7 @@ METRIC = "int8 TOPS & bf16 TFLOPS per GEMM shape, 1 GB300; % of dense tensor-cor
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FLUSH_BYTES = 512 << 20
+CLEAN_READ_BYTES = 256 << 20
 
 
 def load_peaks():
@@ -195,11 +204,18 @@ def run_ours(args, rank, world, dev):
     wl = select(args)
     cases = [GemmCase(g, dev) for g in wl.gemms]
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    clean = torch.ones(CLEAN_READ_BYTES // 4, dtype=torch.float32, device=dev)
+    sink = torch.empty((), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step(times=None, kern=None):
+    def do_flush(i, clean_l2=False):
+        flush.fill_(float(i))
+        if clean_l2:  # read another buffer: the flush's dirty lines are written back now
+            torch.sum(clean, dim=0, out=sink)
+
+    def step(times=None, kern=None, clean_l2=False):
         for i, c in enumerate(cases):
-            flush.fill_(float(i))
+            do_flush(i, clean_l2)
             if times is not None:
                 s, e = times[i]
                 s.record(stream)
@@ -250,6 +266,35 @@ def run_ours(args, rank, world, dev):
     for k in range(args.steps):
         step(None, kev[k])
     torch.cuda.synchronize()
+    # Clean-flush pass: the same steps after a flush that leaves L2 clean.
+    cev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in cases] for _ in range(args.steps)]
+    for k in range(args.steps):
+        step(cev[k], clean_l2=True)
+    torch.cuda.synchronize()
+    # Read ceiling of the HBM-bound GEMMs: a plain read of the same bytes
+    # after the same (dirty) flush (outside the timed steps).
+    peaks, peak_src = load_peaks()
+    bf16_peak = float(peaks.get("bf16_tflops", FALLBACK["bf16_tflops"]))
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK["hbm_gbs"]))
+    read_ms = {}
+    for i, c in enumerate(cases):
+        if bound_of(c.g, bf16_peak, hbm_peak) != "hbm":
+            continue
+        nbytes = compulsory_bytes(c.g) // 16 * 16
+        buf = torch.ones(nbytes // 4, dtype=torch.float32, device=dev)
+        evs = []
+        for k in range(args.steps + 2):
+            do_flush(i)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            G.check(G.gemm_selftest_read_stream(buf, nbytes, stream))
+            b.record(stream)
+            if k >= 2:
+                evs.append((a, b))
+        torch.cuda.synchronize()
+        read_ms[i] = statistics.median(x.elapsed_time(y) for x, y in evs)
+        del buf
     # the timed region is short: keep sampling clocks over the same work for
     # about a second more so the clock record has samples under load
     t1 = time.perf_counter()
@@ -260,6 +305,7 @@ def run_ours(args, rank, world, dev):
 
     per_gemm_ms = [[ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(args.steps)] for i in range(len(cases))]
     per_kern_ms = [[kev[k][i][0].elapsed_time(kev[k][i][1]) for k in range(args.steps)] for i in range(len(cases))]
+    per_clean_ms = [[cev[k][i][0].elapsed_time(cev[k][i][1]) for k in range(args.steps)] for i in range(len(cases))]
     gemm_ms = sum(sum(x) for x in per_gemm_ms) / args.steps  # device ms per step
     ops = sum(c.g.flops for c in cases)
 
@@ -353,19 +399,23 @@ def run_ours(args, rank, world, dev):
 
     gemm_ms, e2e_max, wall = max_over_ranks([gemm_ms, e2e_ms or 0.0, wall], world, dev)
 
-    peaks, peak_src = load_peaks()
-    bf16_peak = float(peaks.get("bf16_tflops", FALLBACK["bf16_tflops"]))
-    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK["hbm_gbs"]))
     per = []
     for i, c in enumerate(cases):
         ms = statistics.median(per_gemm_ms[i])
         kms = statistics.median(per_kern_ms[i])
+        cms = statistics.median(per_clean_ms[i])
         tops = c.g.flops / (ms * 1e-3) / 1e12
         gbps = compulsory_bytes(c.g) / (ms * 1e-3) / 1e9
-        per.append({"gemm": c.g.name, "bound": bound_of(c.g, bf16_peak, hbm_peak), "ms": round(ms, 5),
-                    "main_kernel_ms": round(kms, 5), "tops": round(tops, 2),
-                    "frac_of_bf16_peak": round(tops / bf16_peak, 4), "gbps": round(gbps, 1),
-                    "frac_of_hbm": round(gbps / hbm_peak, 4), "best_ms": round(min(per_gemm_ms[i]), 5)})
+        row = {"gemm": c.g.name, "bound": bound_of(c.g, bf16_peak, hbm_peak), "ms": round(ms, 5),
+               "main_kernel_ms": round(kms, 5), "tops": round(tops, 2),
+               "frac_of_bf16_peak": round(tops / bf16_peak, 4), "gbps": round(gbps, 1),
+               "frac_of_hbm": round(gbps / hbm_peak, 4), "best_ms": round(min(per_gemm_ms[i]), 5),
+               "ms_clean_l2": round(cms, 5),
+               "frac_of_hbm_clean_l2": round(compulsory_bytes(c.g) / (cms * 1e-3) / 1e9 / hbm_peak, 4)}
+        if i in read_ms:
+            row["read_ceiling_ms"] = round(read_ms[i], 5)
+            row["frac_of_read_ceiling"] = round(read_ms[i] / ms, 4)
+        per.append(row)
     # dominant kernel: the main kernel of the GEMM with the largest time
     dom = max(range(len(cases)), key=lambda i: statistics.mean(per_gemm_ms[i]))
     dk_ms = statistics.mean(per_kern_ms[dom])
@@ -390,9 +440,7 @@ def run_ours(args, rank, world, dev):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(gemm_ms, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": dtype_desc(wl), "data": "synthetic (seeded, workloads.py)",
-        "config": {"workload": wl.name, "description": wl.description,
-                   "gemms": [c.g.name for c in cases], "l2": "flushed (512 MiB write) before every timed GEMM",
-                   "parallelism": f"replicas x{world}"},
+        "config": config_of(wl, world),
         "per_gemm": per,
         "roofline": roof,
         "e2e": None if e2e_ms is None else {
@@ -404,6 +452,14 @@ def run_ours(args, rank, world, dev):
         "cpu_baseline": cpu,
     }
     return line
+
+
+def config_of(wl, world):
+    """The `config` object of the JSON line, identical in both arms."""
+    return {"workload": wl.name, "description": wl.description, "gemms": [g.name for g in wl.gemms],
+            "l2": "flushed (512 MiB write) before every timed GEMM; per GEMM also after a clean flush "
+                  "(write, then a 256 MiB read)",
+            "parallelism": f"replicas x{world}"}
 
 
 # Source files that determine each kernel family's code: DRAM counters of a
@@ -561,7 +617,7 @@ def run_reference(args, rank, world):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": dtype_desc(wl).replace("int32", "int64").replace("fp32", "f64") + " (oracle)",
         "data": "synthetic (seeded, workloads.py)",
-        "config": {"workload": wl.name, "description": wl.description, "gemms": [g.name for g in wl.gemms]},
+        "config": config_of(wl, world),
         "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": oracle.num_threads(),
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -706,7 +762,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="square_sweep_512_4096", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--workload", default="all_configs", choices=sorted(W.WORKLOADS))
     ap.add_argument("--gemm", action="append", default=[],
                     help="run only this GEMM of the workload (repeatable), e.g. bf16_4096x4096x4096_Bcol")
     ap.add_argument("--no-e2e", action="store_true")

@@ -34,12 +34,14 @@
  *     GB300_GEMM_PAIR, GB300_GEMM_SPLITS, GB300_GEMM_SKINNY_MAX_M,
  *     GB300_GEMM_TMA_STORE=0, GB300_GEMM_PDL=0, GB300_GEMM_S8TM=0 (int8
  *     GEMMs with one operand of at most 128 rows take the general path
- *     instead of converting the large operand inside the kernel) and
- *     GB300_GEMM_S8A=1 (int8 GEMMs planned as 128 x 224 tiles convert A
- *     inside the kernel instead of staging it; slower, off by default), read
- *     at every call.
+ *     instead of converting the large operand inside the kernel),
+ *     GB300_GEMM_TINY_MAX_MACS (largest M*N*K of an int8 GEMM computed in one
+ *     launch on the CUDA cores; 0 disables that kernel, and so does forcing
+ *     a tile width, family or split with the variables above) and
+ *     GB300_GEMM_DEBUG=1 (prints each plan to stderr).  They are read once,
+ *     at the first call, and again by gemm_reload_overrides().
  *     GB300_GEMM_WAIT_LIMIT_MS (read once) bounds every device-side wait
- *     (default 2000 ms); GB300_GEMM_DEBUG=1 prints each plan to stderr.
+ *     (default 2000 ms).
  */
 #ifndef GB300_GEMM_H
 #define GB300_GEMM_H
@@ -122,8 +124,8 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K,
 
 /*
  * Size of the fixed device scratch array used by gemm_s8s8_s32_noalloc.
- * Every GPU on which the library's device code is loaded holds this much
- * memory until the process exits.
+ * A GPU holds this much memory from the first gemm_s8s8_s32_noalloc call on
+ * it (which loads the array) until the process exits.
  */
 #define GEMM_NOALLOC_SCRATCH_BYTES ((size_t)128 << 20) /* 128 MiB */
 
@@ -137,20 +139,29 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K,
  * convenience of this library.)
  *
  *   Arguments, layouts, results and errors are those of gemm_s8s8_s32, and
- *   the caller still owns A, B and C.  The operands' bf16 staging copies and
+ *   the caller still owns A, B and C.  The results are those of
+ *   gemm_s8s8_s32 bit for bit, but not always its speed: this entry point
+ *   always stages both operands and runs the general tensor-core kernels,
+ *   never the CUDA-core kernel for very small M or the kernel that converts
+ *   a large operand in place.  The operands' bf16 staging copies and
  *   any split-K partial sums live in one static device array of
  *   GEMM_NOALLOC_SCRATCH_BYTES bytes instead of the library's workspace; the
  *   call never calls cudaMalloc, cudaFree or any other allocating routine.
  *   Bytes needed: round256(2*M*K8) + round256(2*K8*N) for column-major B
  *   (round256(2*M*K8) + round256(2*K*N8) for row-major B), plus
  *   round256(4*S*M*N) when the planner splits K into S > 1 parts (S <= 16,
- *   only for problems with fewer output tiles than SMs), where K8 and N8 are
+ *   only for problems with fewer output tiles than SMs, unless
+ *   GB300_GEMM_SPLITS overrides the planner), where K8 and N8 are
  *   K and N rounded up to multiples of 8.  A problem needing more returns
  *   GEMM_ERR_UNSUPPORTED and launches nothing.
  *
- *   The first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress) with that device current and caches it; make that
- *   first call before any stream capture.  All calls share the one array and
+ *   The first call on each device loads the array -- that is the moment the
+ *   GPU gives up its GEMM_NOALLOC_SCRATCH_BYTES -- and looks up its device
+ *   address (cudaGetSymbolAddress) with that device current, then caches it.
+ *   So make that first call (any valid problem will do) before the caller's
+ *   own allocator reserves the device's memory, and before any stream
+ *   capture.  After a cudaDeviceReset() call gemm_release_resources(), which
+ *   forgets the cached address, before the next call.  All calls share the one array and
  *   it keeps whatever the last call left in it; every byte a call reads from
  *   it is written earlier in the same call, so nothing needs clearing.  Calls
  *   whose execution overlaps on the GPU (on different streams, or from
@@ -172,13 +183,21 @@ const char *gemm_status_string(gemm_status_t status);
  */
 gemm_status_t gemm_device_status(void);
 
-/* Frees the workspace and cached state of the current device.  The caller
- * must ensure no library kernel is still running. */
+/* Frees the workspace and cached state (device addresses looked up at the
+ * first call, including the no-allocation scratch's) of the current device.
+ * The caller must ensure no library kernel is still running.  Call it after
+ * a cudaDeviceReset() before using the library on that device again. */
 void gemm_release_resources(void);
 
 /* Number of kernel launches the library has enqueued since load (all
  * devices); lets a caller count the kernels a region of work launched. */
 uint64_t gemm_launch_count(void);
+
+/* Re-reads the planner overrides (GB300_GEMM_BN ... GB300_GEMM_DEBUG, listed
+ * at the top of this file) from the environment; otherwise they are read
+ * once, at the first GEMM call.  A test and benchmark aid (the paper has no
+ * counterpart); calls already enqueued are not affected. */
+void gemm_reload_overrides(void);
 
 /*
  * Failure-detection self-test (a diagnostic; the paper has no counterpart).
@@ -190,6 +209,56 @@ uint64_t gemm_launch_count(void);
  * usable.  Returns GEMM_OK once the probe is launched.
  */
 gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream);
+
+/*
+ * The plan the library would use for a GEMM (a host-only query: no device
+ * is touched, so it also runs on a machine without a GPU).  The planner is
+ * the GB300 restatement of the paper's tile model and balanced-point search
+ * (Sec. 4.5.1 Eq. 1-5, Sec. 4.5.2 Eq. 6-10): among the compiled kernel
+ * variants -- one CTA per 128 x BN tile or a CTA pair per 256 x BN tile --
+ * and K splits it takes the least modelled time, from per-variant costs
+ * fitted to measurements on GB300.
+ *   int8: nonzero for the int8 entry points, 0 for bf16.  b_layout as in
+ *   the GEMM calls.  sms: SMs of the device (152 on GB300); pair_slots:
+ *   co-resident CTA pairs (76).  Operands are taken as tight (lda = K, ldb
+ *   and ldc = N or K) and 16-byte aligned; the planner overrides in force
+ *   (GB300_GEMM_*) apply.
+ *   out->route: GEMM_ROUTE_*; bn: tile width (the small operand's tile
+ *   height for GEMM_ROUTE_SMALL_OPERAND); splits: K split factor; stages:
+ *   pipeline depth of the tensor-core kernel; grid: CTAs launched;
+ *   model_us: modelled time of the tensor-core kernel and split-K reduction.
+ * Returns GEMM_ERR_INVALID_ARG / GEMM_ERR_UNSUPPORTED like the GEMM calls.
+ */
+enum {
+  GEMM_ROUTE_NONE = 0,           /* M == 0 or N == 0: nothing to do */
+  GEMM_ROUTE_ZERO_FILL = 1,      /* K == 0 */
+  GEMM_ROUTE_SMALL_M = 2,        /* CUDA-core kernel for very small M */
+  GEMM_ROUTE_SMALL_OPERAND = 3,  /* int8 with one operand of <= 128 rows, converted in the kernel */
+  GEMM_ROUTE_TC_SINGLE = 4,      /* tensor-core kernel, one CTA per 128 x BN tile */
+  GEMM_ROUTE_TC_PAIR = 5,        /* tensor-core kernel, a CTA pair per 256 x BN tile */
+  GEMM_ROUTE_TINY = 6            /* int8 problem small enough for one CUDA-core launch */
+};
+typedef struct {
+  int route;
+  int bn;
+  int splits;
+  int stages;
+  int grid;
+  double model_us;
+} gemm_plan_t;
+gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_layout, int sms, int pair_slots,
+                              gemm_plan_t *out);
+
+/*
+ * Read-bandwidth diagnostic (the paper has no counterpart): enqueues one
+ * kernel that reads `bytes` of device memory at `ptr` with 16-byte loads
+ * (four blocks per SM, several loads in flight per thread) and discards
+ * them, so that the time between two events around it is what a plain read
+ * of that many bytes takes -- the ceiling an HBM-bound GEMM of the same
+ * traffic could reach.  ptr 16-byte aligned, bytes a multiple of 16, else
+ * GEMM_ERR_INVALID_ARG.  Nothing is written to `ptr`'s buffer.
+ */
+gemm_status_t gemm_selftest_read_stream(const void *ptr, size_t bytes, gemm_stream_t stream);
 
 /*
  * Profiling aid.  With both arguments non-NULL (cudaEvent_t handles created

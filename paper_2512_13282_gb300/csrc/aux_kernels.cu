@@ -280,7 +280,34 @@ __global__ void wait_timeout_probe_kernel(uint32_t *err, uint64_t limit_ns) {
   if (threadIdx.x == 0) (void)mbar_wait(smem_addr(&bar), 0, &abort_flag, err, limit_ns);
 }
 
+// Reads n 16-byte vectors with streaming loads, four in flight per thread,
+// and keeps nothing: the time of a plain read of that many bytes.  The
+// result folds into one word that is written only if it equals a value no
+// read of real data is expected to give, so the loads are not optimised away.
+__global__ void __launch_bounds__(512) read_stream_kernel(const uint4 *__restrict__ p, uint64_t n, uint32_t *sink) {
+  uint32_t acc = 0;
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (; i + 3 * stride < n; i += 4 * stride) {
+    const uint4 a = __ldcs(p + i), b = __ldcs(p + i + stride), c = __ldcs(p + i + 2 * stride),
+                d = __ldcs(p + i + 3 * stride);
+    acc ^= a.x ^ a.w ^ b.y ^ b.x ^ c.z ^ c.y ^ d.w ^ d.z;
+  }
+  for (; i < n; i += stride) {
+    const uint4 a = __ldcs(p + i);
+    acc ^= a.x ^ a.w;
+  }
+  if (acc == 0x9E3779B9u) *sink = acc;
+}
+
 }  // namespace
+
+cudaError_t launch_read_stream(const void *p, size_t bytes, uint32_t *sink, int sms, cudaStream_t st) {
+  const uint64_t n = bytes / 16;
+  if (n == 0) return cudaSuccess;
+  read_stream_kernel<<<(unsigned)(4 * sms), 512, 0, st>>>(static_cast<const uint4 *>(p), n, sink);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStream_t st) {
   wait_timeout_probe_kernel<<<1, 32, 0, st>>>(err, limit_ns);

@@ -14,12 +14,14 @@
 
 #include "gb300_gemm.h"
 #include "gemm_internal.h"
+#include "plan_table.h"
 
 using namespace gb300;
 
-// Device error word: kernels record kDevErrTimeout here when a bounded wait
-// expires.  Read and cleared by gemm_device_status().
-__device__ uint32_t g_gemm_dev_err = 0;
+// Device error word (element 0): kernels record kDevErrTimeout here when a
+// bounded wait expires; read and cleared by gemm_device_status().  Element 1
+// is the sink of the read-bandwidth diagnostic.
+__device__ uint32_t g_gemm_dev_err[2] = {0u, 0u};
 
 namespace {
 
@@ -44,10 +46,66 @@ cudaEvent_t g_prof_start = nullptr, g_prof_stop = nullptr;
 
 }  // namespace
 
-bool gb300::pdl_enabled() {
-  const char *s = std::getenv("GB300_GEMM_PDL");
-  return !(s && std::atoi(s) == 0);
+namespace {
+
+// Test and benchmark overrides of the planner, read from the environment
+// once (at the first call) and again by gemm_reload_overrides():
+// GB300_GEMM_BN (128, 192, 224 or 256) forces the tile width,
+// GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
+// split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
+// CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores, GB300_GEMM_PDL=0
+// plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
+// small-operand shapes, GB300_GEMM_TINY_MAX_MACS the largest
+// int8 problem (M * N * K) sent to the one-launch CUDA-core kernel (0
+// disables it), GB300_GEMM_DEBUG=1 prints each plan.
+struct Overrides {
+  int bn = 0;            // 0: planner's choice
+  int pair = -1;         // -1: planner's choice
+  int splits = 0;        // 0: planner's choice
+  int skinny_max_m = -1; // -1: built-in limit
+  bool tma_store = true;
+  bool pdl = true;
+  bool s8tm = true;
+  int64_t tiny_max_macs = -1;  // -1: built-in limit
+  bool debug = false;
+};
+
+int env_int(const char *name, int dflt) {
+  const char *s = std::getenv(name);
+  return s ? std::atoi(s) : dflt;
 }
+
+Overrides read_overrides() {
+  Overrides o;
+  o.bn = env_int("GB300_GEMM_BN", 0);
+  o.pair = env_int("GB300_GEMM_PAIR", -1);
+  o.splits = env_int("GB300_GEMM_SPLITS", 0);
+  o.skinny_max_m = env_int("GB300_GEMM_SKINNY_MAX_M", -1);
+  o.tma_store = env_int("GB300_GEMM_TMA_STORE", 1) != 0;
+  o.pdl = env_int("GB300_GEMM_PDL", 1) != 0;
+  o.s8tm = env_int("GB300_GEMM_S8TM", 1) != 0;
+  if (const char *t = std::getenv("GB300_GEMM_TINY_MAX_MACS")) o.tiny_max_macs = std::atoll(t);
+  o.debug = env_int("GB300_GEMM_DEBUG", 0) != 0;
+  return o;
+}
+
+std::mutex g_ovr_mu;
+Overrides g_ovr;
+bool g_ovr_loaded = false;
+
+// The overrides in force (a copy, so that a concurrent reload cannot tear it).
+Overrides overrides() {
+  std::lock_guard<std::mutex> lk(g_ovr_mu);
+  if (!g_ovr_loaded) {
+    g_ovr = read_overrides();
+    g_ovr_loaded = true;
+  }
+  return g_ovr;
+}
+
+}  // namespace
+
+bool gb300::pdl_enabled() { return overrides().pdl; }
 
 namespace {
 
@@ -107,20 +165,6 @@ gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
   }
   d.ws_bytes = grown;
   return GEMM_OK;
-}
-
-// Test and benchmark overrides of the planner, read at every call:
-// GB300_GEMM_BN (128, 192, 224 or 256) forces the tile width,
-// GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
-// split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
-// CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores, GB300_GEMM_PDL=0
-// plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
-// small-operand shapes, GB300_GEMM_S8A=1 the int8 kernel that converts A in
-// tensor memory for 224-wide tiles; GB300_GEMM_DEBUG=1 (read once) prints
-// each plan.
-int env_int(const char *name) {
-  const char *s = std::getenv(name);
-  return s ? std::atoi(s) : 0;
 }
 
 // Grow the zeroed ticket counters of the small-M kernel to `count`.
@@ -197,49 +241,60 @@ struct Plan {
   TcVariant v;
   TcParams p;
   int grid;
+  double model_us;  // modelled time of the tensor-core kernel (and split-K reduction)
 };
 
 // Kernel family, tile width, split-K factor and grid for an M x N x K
-// problem on `sms` SMs.
+// problem on `sms` SMs and `pairs` co-resident SM pairs.
 //
-// Tile choice is the GB300 counterpart of the paper's balanced-tile search
-// (Sec. 4.5): the kernel runs in ceil(units / slots) rounds of one unit per
-// slot, where a slot is an SM (single-CTA kernel, 128 x BN tiles) or an SM
-// pair (pair kernel, 256 x BN tiles).  What one round costs was measured on
-// GB300 for long K (bf16, 4096^3..8192^3, relative to a 256 x 256 pair
-// round): it is nearly flat in BN, because the A tile, the pipeline latency
-// and the epilogue are paid by every tile whatever its width.  The family
-// and width with the least rounds * round cost win, the widest on a tie --
-// e.g. 4096^3 with B column-major: single-CTA 128 x 224 tiles in exactly 4
-// rounds of 152; 8192^3: pairs of 256 x 256 tiles.
-//
-// Split K only when the tile count leaves most slots idle and K is long; the
-// reduction then runs as a separate pass over fp32/int32 partials.
-int round_cost(bool pair, int bn) {
-  switch (bn) {
-    case 128: return pair ? 885 : 850;
-    case 192: return pair ? 950 : 920;
-    case 224: return pair ? 1000 : 980;
-    default: return pair ? 1000 : 1070;  // 256
+// The GB300 counterpart of the paper's balanced-tile search (Sec. 4.5).
+// Every candidate -- one CTA per 128 x BN tile or a CTA pair per 256 x BN
+// tile, BN among the compiled widths, K split S ways -- runs in
+// ceil(tiles * S / slots) rounds of one unit per slot (an SM or an SM pair);
+// its modelled time is
+//   max(rounds * (kb_per_unit * kstep + unit), DRAM time) + split terms
+// (Eq. 9 with wave quantisation, Eq. 6-8 and 10), with the per-variant K-step
+// and unit costs and the split constants fitted to measurements on GB300
+// (plan_table.h, generated by tile_model.py).  The least time wins; on a tie
+// the earlier candidate (single CTA before pair, wider before narrower,
+// fewer splits before more).  tile_model.choose_plan is the same rule.
+double modelled_us(int64_t M, int64_t N, int64_t K, bool int8, bool pair, int bn, int64_t splits, int64_t kb_per,
+                   int64_t rounds) {
+  const int wi = bn == 128 ? 0 : bn == 192 ? 1 : bn == 224 ? 2 : 3;
+  const plan_table::StepCost c = plan_table::kCost[int8 ? 1 : 0][pair ? 1 : 0][wi];
+  const double t_comp = (double)rounds * ((double)kb_per * c.kstep_us + c.unit_us);
+  // DRAM bytes: operands (bf16 in the kernel), re-reads of B when neither B
+  // nor both operands stay in L2, C, split-K partials written and read
+  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * K * N;
+  double rb = 1.0;
+  if (!(b_bytes <= plan_table::kL2Bytes / 2 || a_bytes + b_bytes <= plan_table::kL2Bytes)) {
+    rb = (double)ceil_div(M, kBM) / 8.0;
+    if (rb < 1.0) rb = 1.0;
   }
+  const double c_bytes = (double)M * N * (int8 ? 4 : 2) + (splits > 1 ? 8.0 * splits * M * N : 0.0);
+  const double t_mem = (a_bytes + b_bytes * rb + c_bytes) / (plan_table::kHbmGBs * 1e3);
+  double t = t_comp > t_mem ? t_comp : t_mem;
+  if (splits > 1)
+    t += plan_table::kSplitFixedUs[int8 ? 1 : 0] + plan_table::kSplitUsPerMB[int8 ? 1 : 0] * 4.0 * splits * M * N / 1e6;
+  return t;
 }
 
-Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms) {
+Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms, int pairs) {
   Plan pl{};
-  const int pairs = pair_slots();
   static const int kWidthsKMajor[] = {256, 224, 192, 128};
   static const int kWidthsMNMajor[] = {256, 192, 128};
   static const int kPairWidthsMNMajor[] = {256, 128};
-  const int force_bn = env_int("GB300_GEMM_BN");
-  const char *force_pair_s = std::getenv("GB300_GEMM_PAIR");
-  const int force_pair = force_pair_s ? std::atoi(force_pair_s) : -1;
+  const Overrides ovr = overrides();
+  const bool int8 = epi == kEpiS32;
+  const int64_t num_kb = ceil_div(K, kBK);
   bool best_pair = false;
   int best_bn = 128;
-  int64_t best_cost = -1;
+  int64_t best_splits = 1;
+  double best_cost = -1.0;
   for (int fam = 0; fam < 2; ++fam) {
     const bool pair = fam == 1;
     if (pair && (M <= kBM || pairs <= 0)) continue;  // the second CTA would only compute padding
-    if (force_pair >= 0 && (force_pair != 0) != pair) continue;
+    if (ovr.pair >= 0 && (ovr.pair != 0) != pair) continue;
     const int *widths = b_kmajor ? kWidthsKMajor : (pair ? kPairWidthsMNMajor : kWidthsMNMajor);
     const int nw = b_kmajor ? 4 : (pair ? 2 : 3);
     const int64_t slots = pair ? pairs : sms;
@@ -247,13 +302,32 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
     for (int i = 0; i < nw; ++i) {
       const int bn = widths[i];
       if (N <= 128 && bn != 128) continue;
-      if (force_bn > 0 && force_bn != bn) continue;
-      const int64_t rounds = ceil_div(tiles_m * ceil_div(N, bn), slots);
-      const int64_t cost = rounds * round_cost(pair, bn);
-      if (best_cost < 0 || cost < best_cost) {
-        best_cost = cost;
-        best_pair = pair;
-        best_bn = bn;
+      if (ovr.bn > 0 && ovr.bn != bn) continue;
+      const int64_t tiles = tiles_m * ceil_div(N, bn);
+      int64_t seen[17] = {};
+      int nseen = 0;
+      for (int64_t s = 1; s <= 16; ++s) {
+        int64_t kb_per = ceil_div(num_kb, s < num_kb ? s : num_kb);
+        int64_t s2 = ceil_div(num_kb, kb_per);
+        if (ovr.splits >= 1) {  // forced: exactly that split
+          if (s > 1) break;
+          const int64_t f = ovr.splits < num_kb ? ovr.splits : num_kb;
+          kb_per = ceil_div(num_kb, f);
+          s2 = ceil_div(num_kb, kb_per);
+        } else {
+          bool dup = false;
+          for (int j = 0; j < nseen; ++j) dup = dup || seen[j] == s2;
+          if (dup) continue;
+          if (s2 > 1 && (kb_per < 4 || tiles * s2 > 2 * slots)) continue;
+        }
+        seen[nseen++] = s2;
+        const double cost = modelled_us(M, N, K, int8, pair, bn, s2, kb_per, ceil_div(tiles * s2, slots));
+        if (best_cost < 0 || cost < best_cost - 1e-9) {
+          best_cost = cost;
+          best_pair = pair;
+          best_bn = bn;
+          best_splits = s2;
+        }
       }
     }
   }
@@ -263,21 +337,8 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   const int64_t tiles_m = ceil_div(M, pair ? 2 * kBM : kBM);
   const int64_t tiles_n = ceil_div(N, bn);
   const int64_t tiles = tiles_m * tiles_n;
-  const int64_t num_kb = ceil_div(K, kBK);
-  int64_t splits = 1;
-  // A split pays for an extra reduction launch (several microseconds), so
-  // only long reductions (K >= 2048) over few tiles are split, keeping >= 8
-  // k-blocks per split.
-  if (tiles * 2 <= slots && num_kb >= 32) {
-    splits = slots / tiles;
-    if (splits > num_kb / 8) splits = num_kb / 8;
-    if (splits > 16) splits = 16;
-    if (splits < 1) splits = 1;
-  }
-  const int force_splits = env_int("GB300_GEMM_SPLITS");
-  if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
-  const int64_t kb_per = ceil_div(num_kb, splits);
-  splits = ceil_div(num_kb, kb_per);
+  const int64_t kb_per = ceil_div(num_kb, best_splits);
+  const int64_t splits = ceil_div(num_kb, kb_per);
   // Output path: the bf16 224-wide kernels keep a pipeline stage and stage
   // their TMA stores through 1 KB blocks; for int8 at 192/224, TMA stores
   // (4 KB blocks, one stage less) win up to 128 K steps per unit, beyond
@@ -290,6 +351,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   else
     tma_out = ((bn != 224 && bn != 192) || kb_per <= 128) ? 1 : 0;
   pl.v = TcVariant{bn, b_kmajor, epi, pair, tma_out};
+  pl.model_us = best_cost;
   TcParams &p = pl.p;
   p.M = (int)M;
   p.N = (int)N;
@@ -306,14 +368,14 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms)
   const int64_t units = tiles * splits;
   const int64_t used = units < slots ? units : slots;
   pl.grid = (int)(pair ? 2 * used : used);
-  static const bool debug = env_int("GB300_GEMM_DEBUG") != 0;
-  if (debug)
+  if (ovr.debug)
     std::fprintf(stderr,
                  "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d%s tiles=%lldx%lld splits=%lld grid=%d "
-                 "(SMs %d, co-resident pairs %d)\n",
+                 "model %.1f us (SMs %d, co-resident pairs %d)\n",
                  (long long)M, (long long)N, (long long)K, epi == kEpiS32 ? "int8" : "bf16",
-                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn, tma_out == 2 ? " tma-store-1k" : tma_out ? " tma-store" : "", (long long)tiles_m, (long long)tiles_n,
-                 (long long)splits, pl.grid, sms, pairs);
+                 b_kmajor ? "col" : "row", pair ? "pair" : "single", bn,
+                 tma_out == 2 ? " tma-store-1k" : tma_out ? " tma-store" : "", (long long)tiles_m,
+                 (long long)tiles_n, (long long)splits, pl.grid, best_cost, sms, pairs);
   return pl;
 }
 
@@ -343,9 +405,8 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   // C with a 16-byte aligned base and pitch; split-K partials when their
   // pitch (N words) is a multiple of 16 bytes.  int16 / int8 outputs and
   // other cases store directly (GB300_GEMM_TMA_STORE=0 forces that).
-  const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
   const bool s32 = pl.v.epi == kEpiS32;
-  const bool tma_ok = !(tma_env && std::atoi(tma_env) == 0) &&
+  const bool tma_ok = overrides().tma_store &&
                       (p.splits > 1 ? p.N % 4 == 0 && pl.v.tma_out == 1 : p.c_vec != 0);
   // An output that will be stored directly wants the variant with the extra
   // pipeline stage where one exists (int8 at 192 / 224).
@@ -397,6 +458,18 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   return GEMM_OK;
 }
 
+// Largest int8 problem (M * N * K multiply-adds) computed in one launch on
+// the CUDA cores (gemm_tiny.cu) instead of staging + tensor cores: below it
+// the launches, not the arithmetic, set the time.
+constexpr int64_t kTinyMaxMacs = int64_t(1) << 27;  // 512^3
+
+int64_t tiny_max_macs() {
+  const Overrides o = overrides();
+  // a forced tile width, family or split asks for the tensor-core kernels
+  if (o.bn > 0 || o.pair >= 0 || o.splits >= 1) return 0;
+  return o.tiny_max_macs >= 0 ? o.tiny_max_macs : kTinyMaxMacs;
+}
+
 // Largest M sent to the CUDA-core small-M kernel: there every B element is
 // used at most a few times and streaming B once is the cost.  Measured on
 // GB300 against the tensor-core path (N = 4096..11008, K = 4096): int8
@@ -404,11 +477,8 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
 // accumulating with fp32 FMAs, only up to M = 2.
 // GB300_GEMM_SKINNY_MAX_M overrides (0 disables the kernel).
 int skinny_max_m(bool int8) {
-  const char *s = std::getenv("GB300_GEMM_SKINNY_MAX_M");
-  if (s) {
-    const int v = std::atoi(s);
-    return v < 0 ? 0 : (v > 16 ? 16 : v);
-  }
+  const int v = overrides().skinny_max_m;
+  if (v >= 0) return v > 16 ? 16 : v;
   return int8 ? 8 : 2;
 }
 
@@ -470,7 +540,7 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
   if (M <= skinny_max_m(false))
     return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, false, st);
-  Plan pl = make_plan(M, N, K, b_kmajor, kEpiBf16, d->sms);
+  Plan pl = make_plan(M, N, K, b_kmajor, kEpiBf16, d->sms, pair_slots());
   // TMA needs 16-byte aligned bases and row pitches; re-pitch an operand
   // that is not, into the workspace.
   const bool pack_a = !(aligned16(A) && (lda * 2) % 16 == 0);
@@ -508,10 +578,12 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
 
 namespace {
 
-// int8 operand streamed by gemm_s8tm_kernel: K-contiguous rows, boxes of
-// 128 bytes x 128 rows with the 128-byte swizzle its converter warps expect.
-bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t K, uint64_t rows, uint64_t ld) {
-  const cuuint64_t dims[2] = {K, rows};
+// int8 operand streamed by gemm_s8tm_kernel: boxes of 128 bytes x 128 rows
+// with the 128-byte swizzle its converter warps expect.  inner = K and
+// rows = P's rows for a K-contiguous P; inner = P's rows and rows = K for a
+// P stored K x P_rows (read transposed).
+bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t inner, uint64_t rows, uint64_t ld) {
+  const cuuint64_t dims[2] = {inner, rows};
   const cuuint64_t strides[1] = {ld};
   const cuuint32_t box[2] = {128, (cuuint32_t)kBM};
   const cuuint32_t estr[2] = {1, 1};
@@ -520,10 +592,36 @@ bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t K, uint64_t row
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// K splits of the small-operand int8 kernel: enough units to give every SM
+// one, at least 4 k-blocks (of 128) per split, at most 16 (or the forced
+// count); rounded so that no split is empty.
+int64_t s8tm_splits(int64_t tiles, int64_t num_kb, int sms, int forced) {
+  int64_t splits = (int64_t)sms / tiles;
+  if (splits > num_kb / 4) splits = num_kb / 4;
+  if (splits > 16) splits = 16;
+  if (splits < 1) splits = 1;
+  if (forced >= 1) splits = forced < num_kb ? forced : num_kb;
+  return ceil_div(num_kb, ceil_div(num_kb, splits));
+}
+
+// Which operand the small-operand int8 kernel streams, if any: P = B with
+// M <= 128 (swap), P = A with N <= 128 < M; p_kmajor is false for B stored
+// K x N, read transposed.
+bool s8tm_shape(int64_t M, int64_t N, bool b_kmajor, bool *swap, bool *p_kmajor) {
+  if (M <= kBM && N > kBM)
+    *swap = true;
+  else if (N <= kBM && M > kBM)
+    *swap = false;
+  else
+    return false;
+  *p_kmajor = !*swap || b_kmajor;
+  return true;
+}
+
 // Memory-bound int8 shapes, where one operand is far larger than the other:
-// M <= 128 with B stored N x K (the weights, P = B, are streamed as int8 and
-// the activations Q = A staged), or N <= 128 with M > 128 (P = A, Q = B, in
-// either layout).
+// M <= 128 (the weights, P = B, are streamed as int8 and the activations
+// Q = A staged; B stored N x K is read K-major, B stored K x N transposed),
+// or N <= 128 with M > 128 (P = A, Q = B, in either layout).
 // gemm_s8tm_kernel converts P inside the kernel, so P moves once as int8
 // instead of three times as staged bf16.  Returns false, having launched
 // nothing, when the shape or P's alignment (16-byte base and pitch, for
@@ -532,15 +630,10 @@ bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t K, uint64_t row
 bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda, const int8_t *B,
               int64_t ldb, bool b_kmajor, void *C, int64_t ldc, int out_bits, int shift, cudaStream_t st,
               gemm_status_t *status) {
-  const char *env = std::getenv("GB300_GEMM_S8TM");
-  if (env && std::atoi(env) == 0) return false;
-  bool swap;
-  if (b_kmajor && M <= kBM && N > kBM)
-    swap = true;
-  else if (N <= kBM && M > kBM)
-    swap = false;
-  else
-    return false;
+  const Overrides ovr = overrides();
+  if (!ovr.s8tm) return false;
+  bool swap, p_kmajor;  // p_kmajor false: B stored K x N, P's rows are its k-rows
+  if (!s8tm_shape(M, N, b_kmajor, &swap, &p_kmajor)) return false;
   const int8_t *P = swap ? B : A;
   const int64_t ldp = swap ? ldb : lda;
   if (!aligned16(P) || ldp % 16 != 0) return false;
@@ -553,14 +646,8 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   const int64_t num_kb = ceil_div(K, kS8tmKB);
   const int64_t tiles_p = ceil_div(P_rows, kBM), tiles_q = ceil_div(Q_rows, qn);
   const int64_t tiles = tiles_p * tiles_q;
-  int64_t splits = (int64_t)d.sms / tiles;
-  if (splits > num_kb / 4) splits = num_kb / 4;
-  if (splits > 16) splits = 16;
-  if (splits < 1) splits = 1;
-  const int force_splits = env_int("GB300_GEMM_SPLITS");
-  if (force_splits >= 1) splits = force_splits < num_kb ? force_splits : num_kb;
+  int64_t splits = s8tm_splits(tiles, num_kb, d.sms, ovr.splits);
   const int64_t kb_per = ceil_div(num_kb, splits);
-  splits = ceil_div(num_kb, kb_per);
   gemm_status_t s;
   // split-K: int32 outputs are added into C (zeroed by the staging launch),
   // int16 / int8 ones go through int32 partials and the reduction kernel
@@ -578,7 +665,9 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
                           ldc, st) != cudaSuccess)
     return true;
   CUtensorMap tp;
-  if (!encode_s8_rows(&tp, P, (uint64_t)K, (uint64_t)P_rows, (uint64_t)ldp)) return true;
+  if (!(p_kmajor ? encode_s8_rows(&tp, P, (uint64_t)K, (uint64_t)P_rows, (uint64_t)ldp)
+                 : encode_s8_rows(&tp, P, (uint64_t)P_rows, (uint64_t)K, (uint64_t)ldp)))
+    return true;
   S8tmParams p{};
   p.P_rows = (int)P_rows;
   p.Q_rows = (int)Q_rows;
@@ -591,6 +680,7 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   p.splits = (int)splits;
   p.kb_per_split = (int)kb_per;
   p.slab_kb = 1024 / kS8tmKB;
+  p.add_into_c = add_into_c ? 1 : 0;
   p.swap = swap ? 1 : 0;
   p.C = C;
   p.ldc = ldc;
@@ -602,15 +692,15 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   p.q_img = ws;
   const int64_t units = tiles * splits;
   const int grid = (int)(units < d.sms ? units : d.sms);
-  static const bool debug = env_int("GB300_GEMM_DEBUG") != 0;
-  if (debug)
-    std::fprintf(stderr, "[gb300_gemm] M=%lld N=%lld K=%lld int8 s8tm %s QN=%d tiles=%lldx%lld splits=%lld grid=%d\n",
-                 (long long)M, (long long)N, (long long)K, swap ? "swap" : "direct", qn, (long long)tiles_p,
-                 (long long)tiles_q, (long long)splits, grid);
+  if (ovr.debug)
+    std::fprintf(stderr,
+                 "[gb300_gemm] M=%lld N=%lld K=%lld int8 s8tm %s%s QN=%d tiles=%lldx%lld splits=%lld grid=%d\n",
+                 (long long)M, (long long)N, (long long)K, swap ? "swap" : "direct", p_kmajor ? "" : " P-transposed",
+                 qn, (long long)tiles_p, (long long)tiles_q, (long long)splits, grid);
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
   g_launches.fetch_add(1);
-  if (launch_s8tm(qn, tp, p, grid, st) != cudaSuccess) return true;
+  if (launch_s8tm(qn, p_kmajor, tp, p, grid, st) != cudaSuccess) return true;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
   if (splits > 1 && !add_into_c) {
     g_launches.fetch_add(1);
@@ -618,71 +708,6 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
                                  d.sms, st) != cudaSuccess)
       return true;
   }
-  *status = GEMM_OK;
-  return true;
-}
-
-// int8 A of gemm_s8a_kernel: boxes of 64 bytes x 128 rows, 64-byte swizzle.
-bool encode_s8_rows64(CUtensorMap *map, const void *base, uint64_t K, uint64_t rows, uint64_t ld) {
-  const cuuint64_t dims[2] = {K, rows};
-  const cuuint64_t strides[1] = {ld};
-  const cuuint32_t box[2] = {64, (cuuint32_t)kBM};
-  const cuuint32_t estr[2] = {1, 1};
-  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// Compute-bound int8 GEMMs planned as single-CTA 128 x 224 tiles without
-// split-K, with A TMA-legal as int8 (16-byte aligned base and pitch):
-// gemm_s8a_kernel converts A in the kernel, so only B is staged.  Off unless
-// GB300_GEMM_S8A=1: exact, but measured slower than staging both operands
-// (int8 4096^3: 151 against 110 us).  Returns false, having launched
-// nothing, when it is off or the plan or A rules it out.
-bool try_s8a(DeviceState &d, Plan &pl, const int8_t *A, int64_t lda, const int8_t *B, int64_t ldb, bool b_kmajor,
-             void *C, int64_t ldc, int out_esize, cudaStream_t st, gemm_status_t *status) {
-  const char *env = std::getenv("GB300_GEMM_S8A");
-  if (!env || std::atoi(env) != 1) return false;
-  TcParams &p = pl.p;
-  if (pl.v.pair || pl.v.bn != 224 || !b_kmajor || p.splits != 1 || !aligned16(A) || lda % 16 != 0) return false;
-  const int64_t N = p.N, K = p.K;
-  const int64_t ldb_p = (K + 7) / 8 * 8;  // B stored N x K, staged with 16-byte aligned rows
-  gemm_status_t s;
-  if ((s = ensure_workspace(d, align_up((size_t)N * ldb_p * 2, 256), st)) != GEMM_OK) {
-    *status = s;
-    return true;
-  }
-  uint16_t *Bb = static_cast<uint16_t *>(d.ws);
-  *status = GEMM_ERR_CUDA;
-  g_launches.fetch_add(1);
-  if (launch_s8_to_bf16_pair(S8Job{B, N, K, ldb, Bb, ldb_p}, S8Job{nullptr, 0, 0, 0, nullptr, 0}, d.sms, st) !=
-      cudaSuccess)
-    return true;
-  CUtensorMap ta, tb, tout;
-  if (!encode_s8_rows64(&ta, A, (uint64_t)K, (uint64_t)p.M, (uint64_t)lda)) return true;
-  if (!encode_bf16_2d(&tb, Bb, (uint64_t)K, (uint64_t)N, (uint64_t)ldb_p, kBK, 224)) return true;
-  p.C = C;
-  p.ldc = ldc;
-  p.c_vec = aligned16(C) && ((ldc * out_esize) % 16 == 0);
-  p.ws = nullptr;
-  p.out_tma = kOutDirect;
-  tout = ta;
-  const char *tma_env = std::getenv("GB300_GEMM_TMA_STORE");
-  if (p.c_vec && !(tma_env && std::atoi(tma_env) == 0)) {
-    const CUtensorMapDataType type = p.out_bits == 32   ? CU_TENSOR_MAP_DATA_TYPE_INT32
-                                     : p.out_bits == 16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16
-                                                        : CU_TENSOR_MAP_DATA_TYPE_UINT8;
-    if (!encode_out(&tout, type, (uint32_t)out_esize, C, (uint64_t)N, (uint64_t)p.M, (uint64_t)ldc, 1, 32))
-      return true;
-    p.out_tma = kOutTmaC;
-  }
-  p.err = d.err;
-  p.wait_limit_ns = wait_limit_ns();
-  const bool prof = g_prof_start && g_prof_stop;
-  if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
-  g_launches.fetch_add(1);
-  if (launch_s8a(ta, tb, tout, p, pl.grid, st) != cudaSuccess) return true;
-  if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
   *status = GEMM_OK;
   return true;
 }
@@ -709,11 +734,19 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
   if (M <= skinny_max_m(true))
     return run_skinny(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, true, st, out_bits, shift);
+  if ((double)M * (double)N * (double)K <= (double)tiny_max_macs()) {
+    const TinyParams tp{A, lda, B, ldb, C, ldc, M, N, K, out_bits, shift};
+    const bool prof = g_prof_start && g_prof_stop;
+    if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    g_launches.fetch_add(1);
+    if (launch_tiny_s8(tp, !b_kmajor, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    return GEMM_OK;
+  }
   if (try_s8tm(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, out_bits, shift, st, &s)) return s;
-  Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
+  Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms, pair_slots());
   pl.p.out_bits = out_bits;
   pl.p.out_shift = shift;
-  if (try_s8a(*d, pl, A, lda, B, ldb, b_kmajor, C, ldc, out_esize, st, &s)) return s;
   // Stage both operands as bf16 (exact for int8) with 16-byte aligned rows.
   const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
   const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;
@@ -795,9 +828,18 @@ void gemm_release_resources(void) {
   if (d.tickets) cudaFree(d.tickets);
   d.tickets = nullptr;
   d.tickets_count = 0;
+  d.ready = false;  // look the device's symbols up again at the next call
+  noalloc_forget_device(dev);
 }
 
 uint64_t gemm_launch_count(void) { return g_launches.load(); }
+
+void gemm_reload_overrides(void) {
+  const Overrides o = read_overrides();
+  std::lock_guard<std::mutex> lk(g_ovr_mu);
+  g_ovr = o;
+  g_ovr_loaded = true;
+}
 
 gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream) {
   if (limit_ns == 0 || limit_ns > 1000000000ull) return GEMM_ERR_INVALID_ARG;
@@ -806,6 +848,71 @@ gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream
   if (s != GEMM_OK) return s;
   g_launches.fetch_add(1);
   return launch_wait_timeout_probe(d->err, limit_ns, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? GEMM_OK
+             : GEMM_ERR_CUDA;
+}
+
+gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_layout, int sms, int pair_slots_,
+                              gemm_plan_t *out) {
+  if (!out || M < 0 || N < 0 || K < 0 || sms <= 0 || pair_slots_ < 0) return GEMM_ERR_INVALID_ARG;
+  if (b_layout != GEMM_B_ROW_MAJOR_KxN && b_layout != GEMM_B_COL_MAJOR_NxK) return GEMM_ERR_INVALID_ARG;
+  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX || (int8 && K > kMaxExactK)) return GEMM_ERR_UNSUPPORTED;
+  *out = gemm_plan_t{};
+  const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
+  if (M == 0 || N == 0) {
+    out->route = GEMM_ROUTE_NONE;
+    return GEMM_OK;
+  }
+  if (K == 0) {
+    out->route = GEMM_ROUTE_ZERO_FILL;
+    return GEMM_OK;
+  }
+  if (M <= skinny_max_m(int8 != 0)) {
+    out->route = GEMM_ROUTE_SMALL_M;
+    return GEMM_OK;
+  }
+  if (int8 && (double)M * (double)N * (double)K <= (double)tiny_max_macs()) {
+    out->route = GEMM_ROUTE_TINY;
+    out->bn = 32;
+    out->splits = 1;
+    out->grid = (int)(ceil_div(M, 32) * ceil_div(N, 32));
+    return GEMM_OK;
+  }
+  bool swap, p_kmajor;
+  // tight leading dimensions: P's pitch is K (K-major) or N (B stored K x N)
+  if (int8 && overrides().s8tm && s8tm_shape(M, N, b_kmajor, &swap, &p_kmajor) &&
+      (p_kmajor ? K : N) % 16 == 0) {
+    const int64_t Q_rows = swap ? M : N, P_rows = swap ? N : M;
+    const int qn = Q_rows <= 64 ? 64 : 128;
+    const int64_t tiles = ceil_div(P_rows, kBM) * ceil_div(Q_rows, qn);
+    const int64_t splits = s8tm_splits(tiles, ceil_div(K, kS8tmKB), sms, overrides().splits);
+    out->route = GEMM_ROUTE_SMALL_OPERAND;
+    out->bn = qn;
+    out->splits = (int)splits;
+    out->grid = (int)(tiles * splits < sms ? tiles * splits : sms);
+    return GEMM_OK;
+  }
+  const int epi = int8 ? kEpiS32 : kEpiBf16;
+  const Plan pl = make_plan(M, N, K, b_kmajor, epi, sms, pair_slots_);
+  const int ew = int8 && pl.v.bn != 128 ? 8 : 4;
+  out->route = pl.v.pair ? GEMM_ROUTE_TC_PAIR : GEMM_ROUTE_TC_SINGLE;
+  out->bn = pl.v.bn;
+  out->splits = pl.p.splits;
+  out->stages = tc_max_stages(pl.v.pair ? pl.v.bn / 2 : pl.v.bn, ew, pl.v.tma_out);
+  out->grid = pl.grid;
+  out->model_us = pl.model_us;
+  return GEMM_OK;
+}
+
+gemm_status_t gemm_selftest_read_stream(const void *ptr, size_t bytes, gemm_stream_t stream) {
+  if (!ptr || bytes % 16 != 0 || (reinterpret_cast<uintptr_t>(ptr) & 15) != 0) return GEMM_ERR_INVALID_ARG;
+  DeviceState *d = nullptr;
+  gemm_status_t s = device_state(&d);
+  if (s != GEMM_OK) return s;
+  g_launches.fetch_add(1);
+  // the sink sits beside the error word and is written only for one
+  // particular fold of the data
+  return launch_read_stream(ptr, bytes, d->err + 1, d->sms, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
              ? GEMM_OK
              : GEMM_ERR_CUDA;
 }
@@ -843,7 +950,7 @@ gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t
     return launch_zero_fill(C, M, N, ldc, 4, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
   }
   const bool b_kmajor = b_layout == GEMM_B_COL_MAJOR_NxK;
-  Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms);
+  Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms, pair_slots());
   const int64_t b_rows = b_kmajor ? N : K, b_cols = b_kmajor ? K : N;
   const int64_t lda_p = (K + 7) / 8 * 8, ldb_p = (b_cols + 7) / 8 * 8;
   const size_t a_off = 0;

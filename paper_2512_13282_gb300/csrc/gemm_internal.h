@@ -86,6 +86,7 @@ struct S8tmParams {
   int num_kb;        // ceil(K / kS8tmKB)
   int splits, kb_per_split;
   int slab_kb;       // k-blocks per exact fp32 slab (1024 / kS8tmKB)
+  int add_into_c;    // splits add their exact sums into C (int32, zeroed by the Q staging launch)
   int swap;
   void *C;
   int64_t ldc;
@@ -105,14 +106,12 @@ size_t s8tm_q_image_bytes(int qn, int64_t Q_rows, int64_t K);
 cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64_t Q_rows, int64_t K, int qn,
                                 void *img, int32_t *zero_c, int64_t c_rows, int64_t c_cols, int64_t ldc,
                                 cudaStream_t st);
-// qn: 64 or 128 columns of Q per tile.
-cudaError_t launch_s8tm(int qn, const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st);
-
-// int8 GEMM with single-CTA 128 x 224 tiles, A (int8, TMA boxes of 64 x 128)
-// converted in the kernel into TMEM and B staged as bf16, stored N x K
-// (gemm_s8a.cu); p.splits must be 1.
-cudaError_t launch_s8a(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p, int grid,
-                       cudaStream_t st);
+// qn: 64 or 128 columns of Q per tile.  p_kmajor: P's rows are K
+// contiguous (boxes of 128 k x 128 rows); otherwise P's rows are the
+// contiguous dimension of its storage (boxes of 128 rows x 128 k, read
+// transposed by the converters).
+cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const S8tmParams &p, int grid,
+                        cudaStream_t st);
 
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
 // int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is
@@ -127,6 +126,10 @@ cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cuda
 // bf16 copy into an aligned buffer (re-pitching a misaligned operand).
 cudaError_t launch_pack_u16(const uint16_t *src, int64_t rows, int64_t cols, int64_t ld_src,
                             uint16_t *dst, int64_t ld_dst, int sms, cudaStream_t st);
+// Plain streaming read of `bytes` (16-byte aligned, a multiple of 16) with
+// 16-byte loads over 4 blocks per SM; writes `sink` only in a case that does
+// not occur for ordinary data (read-bandwidth diagnostic).
+cudaError_t launch_read_stream(const void *p, size_t bytes, uint32_t *sink, int sms, cudaStream_t st);
 // One-thread kernel whose bounded mbarrier wait is made to expire
 // (failure-detection self-test).
 cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStream_t st);
@@ -145,11 +148,30 @@ cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, i
 gemm_status_t validate_s8(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,
                           int64_t ldb, int b_layout, const void *C, int64_t ldc);
 
+// Forgets the no-allocation scratch address cached for device `dev`
+// (gemm_noalloc.cu).
+void noalloc_forget_device(int dev);
+
 // The int8 GEMM with its staging and split-K scratch in caller-provided
 // device memory of `capacity` bytes (gemm_api.cu; used by gemm_noalloc.cu).
 gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda,
                                    const int8_t *B, int64_t ldb, int b_layout, int32_t *C, int64_t ldc,
                                    cudaStream_t st, void *scratch, size_t capacity);
+
+// Exact int8 GEMM of a small problem in one launch on the CUDA cores
+// (gemm_tiny.cu): 32 x 32 tiles of C, __dp4a over K.
+struct TinyParams {
+  const int8_t *A;
+  int64_t lda;
+  const int8_t *B;
+  int64_t ldb;
+  void *C;
+  int64_t ldc;
+  int64_t M, N, K;
+  int out_bits;   // 32 (int32 C), 16 or 8 (requantised C)
+  int out_shift;  // right shift of requantised outputs, 0..31
+};
+cudaError_t launch_tiny_s8(const TinyParams &p, bool row_b, cudaStream_t st);
 
 // Small-M GEMM on the CUDA cores (gemm_skinny.cu).  M <= 16.
 struct SkinnyParams {

@@ -28,7 +28,9 @@ std::mutex g_mu;
 void *g_scratch_ptr[kMaxDevices] = {};
 
 // Device address of the scratch array on the current device, looked up on
-// the first call per device and cached.
+// the first call per device and cached.  With lazy module loading (CUDA's
+// default) that first lookup is also what loads this file's device code and
+// so reserves the array on the device.
 gemm_status_t scratch_for_current_device(void **out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return GEMM_ERR_CUDA;
@@ -42,6 +44,14 @@ gemm_status_t scratch_for_current_device(void **out) {
   return GEMM_OK;
 }
 }  // namespace
+
+// Forgets the cached scratch address of device `dev` (gemm_release_resources:
+// after a device reset the array is created anew, at another address).
+void gb300::noalloc_forget_device(int dev) {
+  if (dev < 0 || dev >= kMaxDevices) return;
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_scratch_ptr[dev] = nullptr;
+}
 
 extern "C" gemm_status_t gemm_s8s8_s32_noalloc(int64_t M, int64_t N, int64_t K, const int8_t *A,
                                                int64_t lda, const int8_t *B, int64_t ldb, int b_layout,

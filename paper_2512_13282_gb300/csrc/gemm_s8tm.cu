@@ -10,9 +10,11 @@
 // This kernel stages only the small operand and streams the large one as
 // int8:
 //
-//   P  the large operand, int8, K contiguous: B stored N x K when M is
-//      small (P row = column n of C), or A when N is small (P row = row m).
-//      It is the MMA's 128-row A operand, read from TMEM.
+//   P  the large operand, int8: B when M is small (P row = column n of C),
+//      or A when N is small (P row = row m).  It is the MMA's 128-row A
+//      operand, read from TMEM.  P is either K contiguous (A, or B stored
+//      N x K) or P row contiguous (B stored K x N: the TMA box then holds
+//      128 k-rows of 128 P rows, and the converters read it transposed).
 //   Q  the small operand, staged beforehand (s8tm_stage_q_kernel) as the
 //      exact shared-memory image the MMA reads for each (Q tile, k-block):
 //      bf16, K-major, 128-byte swizzled, QN rows x 128 K = QN x 256 bytes,
@@ -111,7 +113,7 @@ template <int QN>
 __device__ __forceinline__ void store_row(const S8tmParams &p, const int32_t (&acc)[QN], int split, int64_t off0,
                                           int64_t step, int64_t q0) {
   const int64_t nq = p.Q_rows - q0;  // valid elements (>= 1)
-  if (p.splits > 1 && p.out_bits == 32) {
+  if (p.add_into_c) {
     // int32 C, zeroed by the Q staging kernel: every split adds its exact
     // partial sums (integer addition, so any order gives the same C)
     int32_t *dst = reinterpret_cast<int32_t *>(p.C) + off0;
@@ -137,7 +139,7 @@ __device__ __forceinline__ void store_row(const S8tmParams &p, const int32_t (&a
   }
 }
 
-template <int QN, int SP, int SQ, int NA>
+template <int QN, int SP, int SQ, int NA, bool PK>
 __global__ void __launch_bounds__(kThreadsS8tm, 1)
     gemm_s8tm_kernel(const __grid_constant__ CUtensorMap tmP, const S8tmParams p) {
   using Cfg = S8tmCfg<QN, SP, SQ, NA>;
@@ -220,7 +222,10 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
           }
           if (is_p) {
             mbar_arrive_expect_tx(pfull_bar(s), kPBytes);
-            tma_load_2d(sP + s * kPBytes, &tmP, kb * kKB, w.tp * kBM, pfull_bar(s));
+            if constexpr (PK)
+              tma_load_2d(sP + s * kPBytes, &tmP, kb * kKB, w.tp * kBM, pfull_bar(s));
+            else
+              tma_load_2d(sP + s * kPBytes, &tmP, w.tp * kBM, kb * kKB, pfull_bar(s));
           } else {
             mbar_arrive_expect_tx(qfull_bar(s), Cfg::kQBytes);
             const uint8_t *q_src = static_cast<const uint8_t *>(p.q_img) +
@@ -317,15 +322,38 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
           break;
         }
         tc_fence_after_sync();
-        const uint32_t row = sP + s * kPBytes + (uint32_t)r * kKB;
-        uint32_t o[64];
+        uint32_t o[64];  // o[c]: bf16 of k = 2c (low half) and 2c + 1
+        if constexpr (PK) {
+          const uint32_t row = sP + s * kPBytes + (uint32_t)r * kKB;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const uint4 v = ld_shared_v4(row + (((uint32_t)j ^ sw) << 4));  // k = 16 j .. 16 j + 15
-          s8x4_to_bf16x4(v.x, o[8 * j + 0], o[8 * j + 1]);
-          s8x4_to_bf16x4(v.y, o[8 * j + 2], o[8 * j + 3]);
-          s8x4_to_bf16x4(v.z, o[8 * j + 4], o[8 * j + 5]);
-          s8x4_to_bf16x4(v.w, o[8 * j + 6], o[8 * j + 7]);
+          for (int j = 0; j < 8; ++j) {
+            const uint4 v = ld_shared_v4(row + (((uint32_t)j ^ sw) << 4));  // k = 16 j .. 16 j + 15
+            s8x4_to_bf16x4(v.x, o[8 * j + 0], o[8 * j + 1]);
+            s8x4_to_bf16x4(v.y, o[8 * j + 2], o[8 * j + 3]);
+            s8x4_to_bf16x4(v.z, o[8 * j + 4], o[8 * j + 5]);
+            s8x4_to_bf16x4(v.w, o[8 * j + 6], o[8 * j + 7]);
+          }
+        } else {
+          // The box holds 128 k-rows of 128 P rows (byte r of k-row k in
+          // chunk (r / 16) ^ (k % 8)).  Lane r reads the 32-bit word holding
+          // its byte from four consecutive k-rows (lanes r, r ^ 1, r ^ 2,
+          // r ^ 3 read the same word; the warp's 32 rows span two chunks, so
+          // the reads are conflict-free) and gathers byte r % 4 of each into
+          // one word of four consecutive k.
+          const uint32_t box = sP + s * kPBytes;
+          const uint32_t rc = (uint32_t)r >> 4, rw = (uint32_t)r & 12u;
+          const uint32_t sel = ((uint32_t)r & 3u) | ((4u + ((uint32_t)r & 3u)) << 4);
+#pragma unroll
+          for (int kq = 0; kq < kKB / 4; ++kq) {
+            uint32_t w4[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const uint32_t k = 4u * kq + i;
+              w4[i] = ld_shared_u32(box + k * 128u + ((rc ^ (k & 7u)) << 4) + rw);
+            }
+            const uint32_t x = __byte_perm(__byte_perm(w4[0], w4[1], sel), __byte_perm(w4[2], w4[3], sel), 0x5410);
+            s8x4_to_bf16x4(x, o[2 * kq], o[2 * kq + 1]);
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(pempty_bar(s));  // this warp's rows of the P box are read
@@ -404,11 +432,21 @@ __global__ void __launch_bounds__(256)
                         int64_t c_rows, int64_t c_cols, int64_t ldc) {
   griddep_launch_dependents();  // the GEMM waits for completion before reading
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= chunks) {  // the remaining threads zero C (int32, split-K by atomic adds)
-    const int64_t total = c_rows * c_cols;
-    for (int64_t e = t - chunks; zero_c && e < total; e += (int64_t)gridDim.x * blockDim.x - chunks) {
-      const int64_t r = e / c_cols;
-      zero_c[r * ldc + (e - r * c_cols)] = 0;
+  if (t >= chunks) {  // the remaining threads zero C (int32, splits added by atomic adds)
+    if (!zero_c) return;
+    // four consecutive elements of a row per step, with one 16-byte store
+    // when the row pitch and base allow it
+    const bool vec = (reinterpret_cast<uintptr_t>(zero_c) & 15) == 0 && (ldc & 3) == 0;
+    const int64_t quads = (c_cols + 3) >> 2, total = c_rows * quads;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x - chunks;
+    for (int64_t e = t - chunks; e < total; e += stride) {
+      const int64_t r = e / quads, c = (e - r * quads) << 2;
+      int32_t *dst = zero_c + r * ldc + c;
+      if (vec && c + 4 <= c_cols) {
+        *reinterpret_cast<int4 *>(dst) = make_int4(0, 0, 0, 0);
+      } else {
+        for (int i = 0; i < 4 && c + i < c_cols; ++i) dst[i] = 0;
+      }
     }
     return;
   }
@@ -438,10 +476,10 @@ __global__ void __launch_bounds__(256)
   img[at] = o;
 }
 
-template <int QN, int SP, int SQ, int NA>
+template <int QN, int SP, int SQ, int NA, bool PK>
 cudaError_t launch_one(const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st) {
   using Cfg = S8tmCfg<QN, SP, SQ, NA>;
-  auto kern = gemm_s8tm_kernel<QN, SP, SQ, NA>;
+  auto kern = gemm_s8tm_kernel<QN, SP, SQ, NA, PK>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmemBytes);
   if (e != cudaSuccess) return e;
   return launch_ex(kern, dim3(grid), dim3(kThreadsS8tm), Cfg::kSmemBytes, st, 1, tp, p);
@@ -459,8 +497,10 @@ cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64
                                 cudaStream_t st) {
   const int64_t num_kb = (K + kKB - 1) / kKB;
   const int64_t chunks = (int64_t)s8tm_q_image_bytes(qn, Q_rows, K) / 16;
-  // 64K more threads zero C when asked (a grid-stride loop over its elements)
-  const int64_t extra = zero_c ? 65536 : 0;
+  // more threads zero C when asked (up to 64K, a grid-stride loop over
+  // four-element pieces of its rows)
+  const int64_t quads = zero_c ? c_rows * ((c_cols + 3) / 4) : 0;
+  const int64_t extra = quads < 65536 ? quads : 65536;
   if (chunks + extra == 0) return cudaSuccess;
   s8tm_stage_q_kernel<<<(unsigned)((chunks + extra + 255) / 256), 256, 0, st>>>(
       src, sq, sk, (int)Q_rows, (int)K, qn, (int)num_kb, static_cast<uint4 *>(img), chunks, zero_c, c_rows, c_cols,
@@ -468,11 +508,13 @@ cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64
   return cudaGetLastError();
 }
 
-cudaError_t launch_s8tm(int qn, const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st) {
+cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const S8tmParams &p, int grid,
+                        cudaStream_t st) {
   // P stages x 16 KB + Q stages x (QN x 256 bytes): 9 x 16 + 2 x 32 KB
   // (QN 128) or 10 x 16 + 3 x 16 KB (QN 64)
-  if (qn == 128) return launch_one<128, 9, 2, 4>(tp, p, grid, st);
-  return launch_one<64, 10, 3, 4>(tp, p, grid, st);
+  if (qn == 128)
+    return p_kmajor ? launch_one<128, 9, 2, 4, true>(tp, p, grid, st) : launch_one<128, 9, 2, 4, false>(tp, p, grid, st);
+  return p_kmajor ? launch_one<64, 10, 3, 4, true>(tp, p, grid, st) : launch_one<64, 10, 3, 4, false>(tp, p, grid, st);
 }
 
 }  // namespace gb300

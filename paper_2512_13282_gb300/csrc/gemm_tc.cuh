@@ -82,6 +82,26 @@ __host__ __device__ constexpr uint32_t pow2_at_least(uint32_t x) {
   return p;
 }
 
+// Shared memory of a tensor-core kernel (the memory constraint of the
+// paper's tile model, Sec. 4.5.1 Eq. 5, on one SM): STAGES operand stages
+// (a 128 x 64 bf16 A box and a bn_cta x 64 B box), the epilogue warps'
+// output staging blocks (4 KB, 1 KB or none each), two barriers per stage
+// and five more, the TMEM address and abort words, and the slack that
+// aligns the ring to 1024 bytes.
+__host__ __device__ constexpr uint32_t tc_smem_bytes(int stages, int bn_cta, int epi_warps, int tma_out) {
+  return (uint32_t)stages * (kABytes + (uint32_t)bn_cta * kRowBytes) +
+         (uint32_t)epi_warps * (tma_out == 1 ? 4096u : tma_out == 2 ? 1024u : 0u) +
+         (uint32_t)(2 * stages + 5) * 8u + 16u + 1024u;
+}
+
+// The deepest pipeline that fits the 227 KB a CTA may use: every compiled
+// kernel takes this many stages.
+__host__ __device__ constexpr int tc_max_stages(int bn_cta, int epi_warps, int tma_out) {
+  int s = 1;
+  while (tc_smem_bytes(s + 1, bn_cta, epi_warps, tma_out) <= 232448u) ++s;
+  return s;
+}
+
 template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 struct TcCfg {
   // MMA N for M = 128 is a multiple of 16 up to 256; the epilogue moves 32
@@ -104,6 +124,7 @@ struct TcCfg {
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
+  static_assert(kSmemBytes == tc_smem_bytes(STAGES, BN, EPI_WARPS, TMA_OUT), "layout and model agree");
   static_assert(kTmemCols <= 512, "TMEM has 512 columns");
 };
 

@@ -109,6 +109,7 @@ struct Tc2Cfg {
   static constexpr uint32_t kNumBars = 2 * STAGES + 4 + 1;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
+  static_assert(kSmemBytes == tc_smem_bytes(STAGES, kHalfN, EPI_WARPS, TMA_OUT), "layout and model agree");
   static_assert(kTmemCols <= 512, "TMEM has 512 columns");
 };
 

@@ -6,19 +6,20 @@ namespace gb300 {
 // Pair tile widths (256 x BN per pair; BN/2 columns of B per CTA): 256 and
 // 128 for either B layout, 224 and 192 for B column-major; TMA stores through
 // 4 KB staging blocks, or 1 KB blocks for 224, which keeps its seventh stage.
+// Every kernel takes the deepest ring that fits (tc_max_stages: 6, 7, 7, 8).
 cudaError_t launch_tc2_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                             const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_pair<256, 6, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 224: return launch_pair<224, 7, true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
-      case 192: return launch_pair<192, 7, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_pair<128, 8, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_pair<256, tc_max_stages(256 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 224: return launch_pair<224, tc_max_stages(224 / 2, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
+      case 192: return launch_pair<192, tc_max_stages(192 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 128: return launch_pair<128, tc_max_stages(128 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_pair<256, 6, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_pair<128, 8, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_pair<256, tc_max_stages(256 / 2, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 128: return launch_pair<128, tc_max_stages(128 / 2, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;
@@ -33,8 +34,9 @@ int pair_slots() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
   if (cached[dev] > 0) return cached[dev];
-  using Cfg = Tc2Cfg<256, 6, true, kEpiBf16, 4, 1>;
-  auto kern = gemm_tc2_kernel<256, 6, true, kEpiBf16, 4, 1>;
+  constexpr int kStages = tc_max_stages(256 / 2, 4, 1);
+  using Cfg = Tc2Cfg<256, kStages, true, kEpiBf16, 4, 1>;
+  auto kern = gemm_tc2_kernel<256, kStages, true, kEpiBf16, 4, 1>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmemBytes) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};

@@ -28,21 +28,21 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 // output path (TMA stores through four 4 KB staging blocks, or, where those
 // would cost a pipeline stage, through four 1 KB blocks of 16 columns):
 // 128 (6, 4 KB), 192 (5, 4 KB), 224 (5, 1 KB; B column-major only), 256
-// (4, 4 KB).
+// (4, 4 KB) -- in each case the deepest ring that fits (tc_max_stages).
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_one<256, 4, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 224: return launch_one<224, 5, true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
-      case 192: return launch_one<192, 5, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_one<128, 6, true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_one<256, tc_max_stages(256, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 224: return launch_one<224, tc_max_stages(224, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
+      case 192: return launch_one<192, tc_max_stages(192, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 128: return launch_one<128, tc_max_stages(128, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_one<256, 4, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 192: return launch_one<192, 5, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_one<128, 6, false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_one<256, tc_max_stages(256, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 192: return launch_one<192, tc_max_stages(192, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 128: return launch_one<128, tc_max_stages(128, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;

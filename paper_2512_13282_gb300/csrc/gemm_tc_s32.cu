@@ -29,25 +29,26 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 // only) and 256 (two warpgroups, 96 / 112 / 128 per thread).  With TMA
 // stores, eight 4 KB staging blocks sit beside the ring (4 stages for
 // 192-256); 192 and 224 also come with 5 stages and direct stores, which
-// long reductions prefer (the planner's choice, v.tma_out).
+// long reductions prefer (the planner's choice, v.tma_out).  Every kernel
+// takes the deepest ring that fits (tc_max_stages).
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
   const bool km = v.b_kmajor, t = v.tma_out != 0;
   switch (v.bn) {
-    case 256: return km ? launch_one<256, 4, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-                        : launch_one<256, 4, false, kEpiS32, 8, 1>(a, b, o, p, grid, st);
+    case 256: return km ? launch_one<256, tc_max_stages(256, 8, 1), true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+                        : launch_one<256, tc_max_stages(256, 8, 1), false, kEpiS32, 8, 1>(a, b, o, p, grid, st);
     case 224:
       if (!km) return cudaErrorInvalidValue;
-      return t ? launch_one<224, 4, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-               : launch_one<224, 5, true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+      return t ? launch_one<224, tc_max_stages(224, 8, 1), true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+               : launch_one<224, tc_max_stages(224, 8, 0), true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
     case 192:
       if (km)
-        return t ? launch_one<192, 4, true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-                 : launch_one<192, 5, true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
-      return t ? launch_one<192, 4, false, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-               : launch_one<192, 5, false, kEpiS32, 8, 0>(a, b, o, p, grid, st);
-    case 128: return km ? launch_one<128, 6, true, kEpiS32, 4, 1>(a, b, o, p, grid, st)
-                        : launch_one<128, 6, false, kEpiS32, 4, 1>(a, b, o, p, grid, st);
+        return t ? launch_one<192, tc_max_stages(192, 8, 1), true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+                 : launch_one<192, tc_max_stages(192, 8, 0), true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+      return t ? launch_one<192, tc_max_stages(192, 8, 1), false, kEpiS32, 8, 1>(a, b, o, p, grid, st)
+               : launch_one<192, tc_max_stages(192, 8, 0), false, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+    case 128: return km ? launch_one<128, tc_max_stages(128, 4, 1), true, kEpiS32, 4, 1>(a, b, o, p, grid, st)
+                        : launch_one<128, tc_max_stages(128, 4, 1), false, kEpiS32, 4, 1>(a, b, o, p, grid, st);
   }
   return cudaErrorInvalidValue;
 }

@@ -28,6 +28,19 @@ GEMM_NOALLOC_SCRATCH_BYTES = 128 << 20
 GEMM_B_ROW_MAJOR_KxN = 0
 GEMM_B_COL_MAJOR_NxK = 1
 
+GEMM_ROUTE_NONE = 0
+GEMM_ROUTE_ZERO_FILL = 1
+GEMM_ROUTE_SMALL_M = 2
+GEMM_ROUTE_SMALL_OPERAND = 3
+GEMM_ROUTE_TC_SINGLE = 4
+GEMM_ROUTE_TC_PAIR = 5
+GEMM_ROUTE_TINY = 6
+
+
+class gemm_plan_t(ctypes.Structure):
+    _fields_ = [("route", ctypes.c_int), ("bn", ctypes.c_int), ("splits", ctypes.c_int),
+                ("stages", ctypes.c_int), ("grid", ctypes.c_int), ("model_us", ctypes.c_double)]
+
 _lock = threading.Lock()
 _lib = None
 
@@ -65,6 +78,12 @@ def library():
         lib.gemm_release_resources.restype = None
         lib.gemm_launch_count.argtypes = []
         lib.gemm_launch_count.restype = ctypes.c_uint64
+        lib.gemm_reload_overrides.argtypes = []
+        lib.gemm_reload_overrides.restype = None
+        lib.gemm_plan_query.argtypes = [i64, i64, i64, ci, ci, ci, ci, ctypes.POINTER(gemm_plan_t)]
+        lib.gemm_plan_query.restype = ci
+        lib.gemm_selftest_read_stream.argtypes = [vp, ctypes.c_size_t, vp]
+        lib.gemm_selftest_read_stream.restype = ci
         lib.gemm_selftest_wait_timeout.argtypes = [ctypes.c_uint64, vp]
         lib.gemm_selftest_wait_timeout.restype = ci
         lib.gemm_profile_events.argtypes = [vp, vp]
@@ -139,9 +158,29 @@ def gemm_launch_count() -> int:
     return int(library().gemm_launch_count())
 
 
+def gemm_reload_overrides() -> None:
+    """Re-read the GB300_GEMM_* planner overrides from the environment."""
+    library().gemm_reload_overrides()
+
+
 def gemm_selftest_wait_timeout(limit_ns: int, stream=None) -> int:
     """Launch the bounded-wait probe that is made to time out; see the header."""
     return int(library().gemm_selftest_wait_timeout(int(limit_ns), _stream(stream)))
+
+
+def gemm_plan_query(M, N, K, int8, b_layout, sms=152, pair_slots=76):
+    """(status, plan) of the host-only planner query; plan is a dict with
+    route, bn, splits, stages, grid and model_us."""
+    out = gemm_plan_t()
+    st = int(library().gemm_plan_query(M, N, K, 1 if int8 else 0, int(b_layout), int(sms), int(pair_slots),
+                                       ctypes.byref(out)))
+    return st, {f: getattr(out, f) for f, _ in gemm_plan_t._fields_}
+
+
+def gemm_selftest_read_stream(ptr, nbytes, stream=None) -> int:
+    """Enqueue the read-bandwidth diagnostic: a plain read of `nbytes` at
+    `ptr` (device memory), results discarded; see the header."""
+    return int(library().gemm_selftest_read_stream(_ptr(ptr), int(nbytes), _stream(stream)))
 
 
 def gemm_profile_events(start_event, stop_event) -> None:

@@ -123,6 +123,17 @@ WORKLOADS = {
 }
 
 
+# The five benchmark configurations in one step, in the order listed above.
+BENCHMARK_CONFIGS = ("int8_square_256", "square_sweep_512_4096", "square_8192", "transformer_projections",
+                     "irregular_skinny")
+WORKLOADS["all_configs"] = Workload(
+    "all_configs",
+    "every GEMM of the five benchmark configurations: int8 256^3 (seed 0); square sweep 512..4096 "
+    "both paths (seed 1); 8192^3 both paths (seed 2); transformer projections (seed 3); irregular "
+    "and skinny shapes (seed 4)",
+    tuple(g for name in BENCHMARK_CONFIGS for g in WORKLOADS[name].gemms))
+
+
 def roofline_sweep_sizes(points: int = 420, seed: int = 5, step: int = 256, largest: int = 8192):
     """(M, N, K) triples of the roofline sweep: the paper sweeps more than
     400 sizes per B layout, each a multiple of the native GEMM size, up to

@@ -62,6 +62,7 @@ def run(dtype, A, B, layout, lda=None, ldb=None, ldc=None, a_off=0, b_off=0, c_o
         cbuf = torch.full((c_off + (M + 2) * ldc + 16,), SENTINEL16, dtype=torch.int16, device="cuda")
         fn, sent = G.gemm_bf16_f32acc_bf16, SENTINEL16
     pc = cbuf.data_ptr() + c_off * cbuf.element_size()
+    G.gemm_reload_overrides()  # the test may have changed GB300_GEMM_* since the last call
     st = fn(M, N, K, pa, lda, pb, ldb, layout, pc, ldc, stream)
     assert st == expect, f"status {st} ({G.gemm_status_string(st)}), expected {expect}"
     torch.cuda.synchronize()

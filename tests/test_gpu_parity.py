@@ -46,9 +46,31 @@ def _check(dtype, A, B, layout, C):
         ok = oracle.bf16_within_bound(C, ref, mag)
         bad = np.argwhere(~ok)
         assert bad.size == 0, f"{len(bad)} out of bound, first at {bad[:5].tolist()}"
-        # diagnostic: most elements are the correctly rounded exact sum
-        exact = np.mean(C == oracle.rne_bf16(ref)) if C.size else 1.0
-        assert exact > 0.5, f"only {exact:.3f} of elements correctly rounded"
+        _check_rounding(C, ref)
+
+
+def _bf16_order(bits):
+    """bf16 bit patterns as integers in the order of their values (adjacent
+    representable values differ by 1)."""
+    b = bits.astype(np.int64)
+    return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+
+def _check_rounding(C, ref):
+    """With fp32 accumulation and one rounding, nearly every element is the
+    correctly rounded exact sum and the rest are one bf16 step from it (sums
+    that lie within the fp32 error of a rounding boundary, or cancel to far
+    below their terms).  A kernel that truncated, rounded twice or dropped a
+    term would leave many elements one step off or more."""
+    want = oracle.rne_bf16(ref)
+    fin = np.isfinite(ref) & np.isfinite(oracle.bf16_bits_to_f64(C))
+    if not fin.any():
+        return
+    steps = np.abs(_bf16_order(C[fin]) - _bf16_order(want[fin]))
+    exact = np.mean(steps == 0)
+    far = np.mean(steps > 1)
+    assert exact >= 0.95, f"only {exact:.4f} of elements are the correctly rounded sum"
+    assert far <= 0.005, f"{far:.4f} of elements are more than one bf16 step from the correctly rounded sum"
 
 
 SHAPES = [
@@ -57,10 +79,15 @@ SHAPES = [
 ]
 
 
-@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("dtype", ["int8", "bf16", "int8-tensor"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M,N,K", SHAPES, ids=[f"{m}x{n}x{k}" for m, n, k in SHAPES])
-def test_parity_shapes(dtype, layout, M, N, K):
+def test_parity_shapes(dtype, layout, M, N, K, monkeypatch):
+    """As routed by the planner (int8 problems this small run in one launch
+    on the CUDA cores), and int8 on the tensor-core kernels (forced)."""
+    if dtype == "int8-tensor":
+        dtype = "int8"
+        monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", "0")
     A, B = _inputs(dtype, M, N, K, layout, seed=M * 7 + N * 3 + K)
     C = U.run(dtype, A, B, layout)
     _check(dtype, A, B, layout, C)
@@ -188,15 +215,18 @@ def test_launch_counter_advances():
 
 # ------------------------------------------------ full-size configurations
 
-def _sample_positions(M, N, BN=256, per_tile=3, cap=12000, seed=0):
-    """Tile corners and edges plus random interior points."""
+def _sample_positions(M, N, BN=128, BMt=128, cap=12000, seed=0):
+    """Tile corners and edges (tiles of BMt rows x BN columns, plus the
+    128-row and 128-column grid) and random interior points."""
     rng = np.random.default_rng(seed)
     rows = set()
-    for r0 in range(0, M, 128):
-        rows.update({r0, min(r0 + 127, M - 1)})
+    for step in {128, BMt}:
+        for r0 in range(0, M, step):
+            rows.update({r0, min(r0 + step - 1, M - 1)})
     cols = set()
-    for c0 in range(0, N, 128):
-        cols.update({c0, min(c0 + 127, N - 1)})
+    for step in {128, BN}:
+        for c0 in range(0, N, step):
+            cols.update({c0, min(c0 + step - 1, N - 1)})
     rows, cols = np.array(sorted(rows)), np.array(sorted(cols))
     rr, cc = np.meshgrid(rows, cols, indexing="ij")
     r = np.concatenate([rr.ravel(), rng.integers(0, M, cap // 2), [M - 1]])
@@ -207,16 +237,45 @@ def _sample_positions(M, N, BN=256, per_tile=3, cap=12000, seed=0):
     return r.astype(np.int64), c.astype(np.int64)
 
 
-FULL = [g for w in W.WORKLOADS.values() for g in w.gemms]
+WHOLE = [g for w in ("int8_square_256", "square_sweep_512_4096", "irregular_skinny") for g in W.WORKLOADS[w].gemms]
 
 
-@pytest.mark.parametrize("g", FULL, ids=[g.name for g in FULL])
-def test_full_size_configs_sampled(g):
-    """Every GEMM of every workload at full size, in the launch configuration
-    the benchmark times: sampled outputs against the oracle, one by one."""
+@pytest.mark.parametrize("g", WHOLE, ids=[g.name for g in WHOLE])
+def test_full_size_configs_whole(g):
+    """The 256^3, square sweep (512^3 .. 4096^3, both paths) and irregular /
+    skinny GEMMs at full size, in the launch configuration the benchmark
+    times: every element against the oracle (int8 bit for bit, bf16 within
+    the bound and correctly rounded)."""
     A, B = W.make_inputs(g)
     C = U.run(g.dtype, A, B, g.layout, shift=g.shift)
-    r, c = _sample_positions(g.M, g.N, seed=g.M + g.N + g.K)
+    _check(g.dtype, A, B, g.layout, C)
+
+
+def _plan_tiles(g):
+    """(rows, columns) of the output tiles the planner uses for g."""
+    st, plan = G.gemm_plan_query(g.M, g.N, g.K, g.int8_in, g.layout)
+    assert st == 0
+    if plan["route"] == G.GEMM_ROUTE_TC_PAIR:
+        return 256, plan["bn"]
+    if plan["route"] == G.GEMM_ROUTE_TC_SINGLE:
+        return 128, plan["bn"]
+    return 128, 128
+
+
+SAMPLED = [g for w in ("square_8192", "transformer_projections", "reduced_precision_outputs")
+           for g in W.WORKLOADS[w].gemms]
+
+
+@pytest.mark.parametrize("g", SAMPLED, ids=[g.name for g in SAMPLED])
+def test_full_size_configs_sampled(g):
+    """The 8192^3, transformer projection and reduced-precision GEMMs at full
+    size, in the launch configuration the benchmark times: outputs at the
+    corners and edges of the tiles the planner chose (e.g. 224 columns, 256
+    rows per CTA pair) and at random points, against the oracle one by one."""
+    A, B = W.make_inputs(g)
+    C = U.run(g.dtype, A, B, g.layout, shift=g.shift)
+    bm, bn = _plan_tiles(g)
+    r, c = _sample_positions(g.M, g.N, BN=bn, BMt=bm, seed=g.M + g.N + g.K)
     if g.int8_in:
         want = oracle.gemm_s8_entries(A, B, g.layout, r, c)
         if g.dtype != "int8":
@@ -226,6 +285,7 @@ def test_full_size_configs_sampled(g):
     else:
         ref, mag = oracle.gemm_bf16_entries(A, B, g.layout, r, c)
         assert oracle.bf16_within_bound(C[r, c], ref, mag).all()
+        _check_rounding(C[r, c], ref)
 
 
 @pytest.mark.parametrize("dtype", ["int8", "bf16"])
@@ -289,6 +349,47 @@ def test_small_m_int8_extremes(monkeypatch):
         assert (C == 2147467264).all()
 
 
+# ------------------------------------- int8 problems in one CUDA-core launch
+
+TINY = [(1, 1, 1), (9, 33, 65), (33, 65, 77), (256, 256, 256), (512, 512, 512), (200, 300, 500), (100, 700, 1001),
+        (40, 50, 6000)]
+
+
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("M,N,K", TINY, ids=[f"{m}x{n}x{k}" for m, n, k in TINY])
+def test_int8_tiny_problems(layout, M, N, K, monkeypatch):
+    """Small int8 problems in one launch of the CUDA-core tile kernel (dp4a,
+    row-major B byte-transposed on the fly): ragged 32 x 32 tiles and K
+    chunks, bit-exact against the oracle."""
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    G.gemm_reload_overrides()
+    A, B = _inputs("int8", M, N, K, layout, seed=M + 3 * N + K)
+    st, plan = G.gemm_plan_query(M, N, K, True, layout)
+    assert plan["route"] == G.GEMM_ROUTE_TINY
+    C = U.run("int8", A, B, layout)
+    _check("int8", A, B, layout, C)
+
+
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+def test_int8_tiny_kernel_forced_misaligned_and_extreme(layout, monkeypatch):
+    """Forced onto larger and misaligned problems: odd leading dimensions and
+    bases (scalar loads), requantised outputs, and K = 131071 of all -128."""
+    monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", str(1 << 40))
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    M, N, K = 300, 333, 2049
+    A, B = _inputs("int8", M, N, K, layout, seed=5)
+    bcols = N if layout == ROW else K
+    C = U.run("int8", A, B, layout, lda=K + 3, ldb=bcols + 1, ldc=N + 2, a_off=1, b_off=3, c_off=1)
+    _check("int8", A, B, layout, C)
+    for out, shift in (("int8_int16", 9), ("int8_int8", 17)):
+        C = U.run(out, A, B, layout, shift=shift)
+        want = oracle.requantize(oracle.gemm_s8(A, B, layout), shift, 16 if out == "int8_int16" else 8)
+        assert np.array_equal(C.astype(np.int64), want)
+    A = np.full((40, 131071), -128, np.int8)
+    B = np.full((131071, 48) if layout == ROW else (48, 131071), -128, np.int8)
+    assert (U.run("int8", A, B, layout) == 2147467264).all()
+
+
 # ------------------------------------------- int8 operand staging variants
 
 STAGING = [(300, 520, 256), (1000, 1500, 3000), (257, 129, 4096), (640, 2048, 784), (2048, 2048, 2048),
@@ -303,6 +404,7 @@ def test_int8_staging_with_and_without_programmatic_launch(layout, M, N, K, pdl,
     otherwise) followed by the GEMM, launched with and without programmatic
     dependent launch: bit-exact either way."""
     monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", "0")
     monkeypatch.setenv("GB300_GEMM_PDL", pdl)
     A, B = _inputs("int8", M, N, K, layout, seed=M ^ N ^ K)
     C = U.run("int8", A, B, layout)
@@ -326,6 +428,7 @@ def test_int8_back_to_back_calls(monkeypatch):
         abuf, pa, lda = U.to_device(A)
         bbuf, pb, ldb = U.to_device(B)
         C = torch.empty((M, N), dtype=torch.int32, device="cuda")
+        G.gemm_reload_overrides()
         assert G.gemm_s8s8_s32(M, N, K, pa, lda, pb, ldb, layout, C, N) == G.GEMM_OK
         keep.append((A, B, layout, abuf, bbuf, C))
     torch.cuda.synchronize()
@@ -340,6 +443,10 @@ S8TM = [
     # M <= 128, B stored N x K: the weights are streamed as int8 (swap)
     (16, 512, 4096, COL), (128, 4096, 1000, COL), (100, 1000, 3000, COL), (64, 300, 64, COL),
     (9, 129, 1024, COL), (128, 1500, 8192, COL),
+    # M <= 128, B stored K x N (N a multiple of 16, so its rows are TMA-legal):
+    # the weights are streamed as int8 and read transposed by the converters
+    (16, 512, 4096, ROW), (128, 4096, 1000, ROW), (100, 1008, 3000, ROW), (64, 304, 64, ROW),
+    (9, 144, 1024, ROW), (128, 1520, 8192, ROW), (17, 160, 1000, ROW),
     # N <= 128, M > 128: A is streamed as int8, B (either layout) staged
     (1000, 64, 3008, ROW), (300, 128, 4096, COL), (2000, 17, 1024, ROW), (129, 100, 2048, COL),
     (640, 65, 11008, ROW),
@@ -351,8 +458,9 @@ S8TM = [
 @pytest.mark.parametrize("splits", ["auto", "1", "3"])
 def test_int8_converted_in_kernel(M, N, K, layout, splits, monkeypatch):
     """The int8 kernel that converts its large operand to bf16 in tensor
-    memory (swap for small M, direct for small N): ragged tiles in every
-    dimension, forced split-K, bit-exact against the oracle."""
+    memory (swap for small M, with B read K-major or transposed; direct for
+    small N): ragged tiles in every dimension, forced split-K, bit-exact
+    against the oracle."""
     if splits != "auto":
         monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
     A, B = _inputs("int8", M, N, K, layout, seed=M * 5 + N + K)
@@ -360,7 +468,8 @@ def test_int8_converted_in_kernel(M, N, K, layout, splits, monkeypatch):
     _check("int8", A, B, layout, C)
 
 
-@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (300, 128, 4096, ROW)], ids=["swap", "direct"])
+@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (16, 512, 4096, ROW), (300, 128, 4096, ROW)],
+                         ids=["swap", "swap-transposed", "direct"])
 @pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("shift", [0, 7, 12])
 def test_int8_converted_in_kernel_requantised(M, N, K, layout, out, shift):
@@ -384,9 +493,19 @@ def test_int8_converted_in_kernel_extremes(monkeypatch):
     monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
     A1, B1 = _inputs("int8", 1, 700, 640, COL, seed=3)
     _check("int8", A1, B1, COL, U.run("int8", A1, B1, COL))
+    # B stored K x N, read transposed: M = 1..8 (normally the CUDA-core
+    # kernel's), all -128 and the largest exact K
+    for M in (1, 2, 5, 8):
+        A1, B1 = _inputs("int8", M, 272, 1100, ROW, seed=M)
+        _check("int8", A1, B1, ROW, U.run("int8", A1, B1, ROW))
+    A = np.full((16, 131071), -128, np.int8)
+    B = np.full((131071, 160), -128, np.int8)
+    assert (U.run("int8", A, B, ROW) == 2147467264).all()
 
 
-@pytest.mark.parametrize("M,N,K,layout", [(128, 4096, 4096, COL), (8192, 64, 8192, ROW)], ids=["swap", "direct"])
+@pytest.mark.parametrize("M,N,K,layout", [(128, 4096, 4096, COL), (128, 11008, 4096, COL), (16, 4096, 4096, ROW),
+                                          (8192, 64, 8192, ROW)],
+                         ids=["swap", "swap-wide", "swap-transposed", "direct"])
 def test_int8_converted_in_kernel_matches_general_path(M, N, K, layout, monkeypatch):
     """Full-size shapes of the benchmark: the new path and the general
     (staged) path give the same int32 results, and sampled entries match the
@@ -400,8 +519,9 @@ def test_int8_converted_in_kernel_matches_general_path(M, N, K, layout, monkeypa
     assert np.array_equal(C1[r, c].astype(np.int64), oracle.gemm_s8_entries(A, B, layout, r, c))
 
 
-@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (100, 1000, 3000, COL), (1000, 64, 3008, ROW)],
-                         ids=["swap", "swap-ragged", "direct"])
+@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (100, 1000, 3000, COL), (1000, 64, 3008, ROW),
+                                          (100, 1008, 3000, ROW)],
+                         ids=["swap", "swap-ragged", "direct", "swap-transposed"])
 @pytest.mark.parametrize("splits", ["3", "8"])
 def test_int8_converted_in_kernel_split_into_padded_c(M, N, K, layout, splits, monkeypatch):
     """Split-K of int32 outputs on the small-operand path adds every split's
@@ -411,27 +531,3 @@ def test_int8_converted_in_kernel_split_into_padded_c(M, N, K, layout, splits, m
     A, B = _inputs("int8", M, N, K, layout, seed=M + K)
     C = U.run("int8", A, B, layout, ldc=N + 5, c_off=3)
     _check("int8", A, B, layout, C)
-
-
-# ---------------- int8 compute-bound tiles with A converted in tensor memory
-
-@pytest.mark.parametrize("M,N,K", [(300, 700, 1504), (130, 450, 3008), (1000, 2000, 4096), (2048, 4096, 1024)],
-                         ids=["ragged", "two-slab-tail", "mid", "wide"])
-@pytest.mark.parametrize("out", ["int8", "int8_int16"])
-def test_int8_a_converted_in_kernel(M, N, K, out, monkeypatch):
-    """Single-CTA 128 x 224 tiles without split-K and an aligned A, with the
-    kernel that converts A in TMEM turned on (GB300_GEMM_S8A=1; it is off by
-    default): A is streamed as int8, only B is staged.  Bit-exact against the
-    oracle and equal to the staged path."""
-    monkeypatch.setenv("GB300_GEMM_BN", "224")
-    monkeypatch.setenv("GB300_GEMM_PAIR", "0")
-    monkeypatch.setenv("GB300_GEMM_SPLITS", "1")
-    monkeypatch.setenv("GB300_GEMM_S8A", "1")
-    A, B = _inputs("int8", M, N, K, COL, seed=M + N)
-    C = U.run(out, A, B, COL, shift=7)
-    if out == "int8":
-        _check("int8", A, B, COL, C)
-    else:
-        assert np.array_equal(C.astype(np.int64), oracle.requantize(oracle.gemm_s8(A, B, COL), 7, 16))
-    monkeypatch.setenv("GB300_GEMM_S8A", "0")
-    assert np.array_equal(U.run(out, A, B, COL, shift=7), C)

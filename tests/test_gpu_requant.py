@@ -52,7 +52,10 @@ SHAPES = [(1, 1, 1), (5, 7, 3), (129, 257, 65), (300, 520, 200), (1000, 1500, 30
 @pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M,N,K", SHAPES, ids=[f"{m}x{n}x{k}" for m, n, k in SHAPES])
-def test_requant_parity_shapes(out, layout, M, N, K):
+@pytest.mark.parametrize("path", ["auto", "tensor"])
+def test_requant_parity_shapes(out, layout, M, N, K, path, monkeypatch):
+    if path == "tensor":
+        monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", "0")
     A, B = _inputs(M, N, K, layout, seed=M + 5 * N + 7 * K)
     shift = _shift_for(out, K)
     C = U.run(out, A, B, layout, shift=shift)
@@ -113,9 +116,12 @@ def test_requant_small_m(out, layout, M, N, K):
 @pytest.mark.parametrize("out", ["int8_int16", "int8_int8"])
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 @pytest.mark.parametrize("M", [4, 300])
-def test_requant_unaligned_c(out, layout, M):
+@pytest.mark.parametrize("path", ["auto", "tensor"])
+def test_requant_unaligned_c(out, layout, M, path, monkeypatch):
     # odd ldc and a C base 1 element past an aligned address: every row
     # starts at a different alignment, so all store widths are used
+    if path == "tensor":
+        monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", "0")
     A, B = _inputs(M, 517, 640, layout, seed=M)
     shift = _shift_for(out, 640)
     C = U.run(out, A, B, layout, ldc=523, c_off=1, shift=shift)
