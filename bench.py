@@ -468,6 +468,7 @@ KERNEL_FAMILIES = {
     "tc": ("gemm_tc.cuh", "gemm_tc2.cuh", "ptx.cuh"),
     "s8tm": ("gemm_s8tm.cu", "ptx.cuh"),
     "skinny": ("gemm_skinny.cu", "ptx.cuh"),
+    "tiny": ("gemm_tiny.cu",),
 }
 
 
