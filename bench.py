@@ -13,7 +13,11 @@ every GEMM again after a clean flush (the same write, then a 256 MiB read of
 another buffer) and reports both per GEMM.  For HBM-bound GEMMs, the time of
 a plain read of the same compulsory bytes after the same flush (the
 library's read-bandwidth diagnostic: 16-byte loads, nothing kept) is measured
-beside it: the ceiling an isolated call of that size can reach.
+beside it: the ceiling an isolated call of that size can reach.  HBM-bound
+GEMMs are also timed back to back (`ms_stream`): R calls on R distinct copies
+of the operands, R x the compulsory bytes >= 384 MB (inputs larger than L2,
+no flush), between one pair of events -- the per-call time a loop of such
+GEMMs sees once launches overlap.
 
   value       whole-job throughput, sum(2*M*N*K) / sum(event time), in TOPS
               (tera-ops/s; int8 MACs and bf16 FMAs both count 2 ops)
@@ -60,6 +64,7 @@ METRIC = "int8 TOPS & bf16 TFLOPS per GEMM shape, 1 GB300; % of dense tensor-cor
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FLUSH_BYTES = 512 << 20
+STREAM_BYTES = 384 << 20
 CLEAN_READ_BYTES = 256 << 20
 
 
@@ -189,6 +194,40 @@ class GemmCase:
         if st != 0:
             raise RuntimeError(f"{g.name} rows {r0}..{r1}: {self.G.gemm_status_string(st)}")
 
+    def time_back_to_back(self, stream, min_bytes, reps=5):
+        """(median ms per call, copies): R calls back to back on R distinct
+        device copies of A, B and C with R x compulsory bytes >= min_bytes,
+        so that each call finds its operands outside L2 without a flush
+        between calls; checked against the single call's result."""
+        g = self.g
+        copies = int(max(3, min(64, -(-min_bytes // max(1, compulsory_bytes(g))))))
+        As = [self.A.clone() for _ in range(copies)]
+        Bs = [self.B.clone() for _ in range(copies)]
+        Cs = [torch.empty_like(self.C) for _ in range(copies)]
+        for r in range(copies):  # untimed: plans and workspace settle
+            self.launch(As[r], Bs[r], Cs[r])
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for r in range(copies):
+                self.launch(As[r], Bs[r], Cs[r])
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b) / copies)
+        self.launch()
+        torch.cuda.synchronize()
+        if g.dtype == "bf16":
+            x, y = Cs[-1].view(torch.bfloat16).float(), self.C.view(torch.bfloat16).float()
+            same = bool(torch.all((x - y).abs() <= 2.0 ** -7 * torch.maximum(x.abs(), y.abs())))
+        else:
+            same = torch.equal(Cs[-1], self.C)
+        if not same:
+            raise RuntimeError(f"{g.name}: back-to-back result differs from the single call")
+        del As, Bs, Cs
+        return statistics.median(ts), copies
+
     def launch_e2e(self):
         self.A.copy_(self.hA, non_blocking=True)
         self.B.copy_(self.hB, non_blocking=True)
@@ -295,6 +334,13 @@ def run_ours(args, rank, world, dev):
         torch.cuda.synchronize()
         read_ms[i] = statistics.median(x.elapsed_time(y) for x, y in evs)
         del buf
+    # Back-to-back pass of the HBM-bound GEMMs (outside the timed steps):
+    # R calls on R distinct operand copies whose bytes together exceed L2.
+    stream_ms = {}
+    if not args.no_stream:
+        for i, c in enumerate(cases):
+            if bound_of(c.g, bf16_peak, hbm_peak) == "hbm":
+                stream_ms[i] = c.time_back_to_back(stream, STREAM_BYTES)
     # the timed region is short: keep sampling clocks over the same work for
     # about a second more so the clock record has samples under load
     t1 = time.perf_counter()
@@ -412,6 +458,11 @@ def run_ours(args, rank, world, dev):
                "frac_of_hbm": round(gbps / hbm_peak, 4), "best_ms": round(min(per_gemm_ms[i]), 5),
                "ms_clean_l2": round(cms, 5),
                "frac_of_hbm_clean_l2": round(compulsory_bytes(c.g) / (cms * 1e-3) / 1e9 / hbm_peak, 4)}
+        if i in stream_ms:
+            t_stream, copies = stream_ms[i]
+            row["ms_stream"] = round(t_stream, 5)
+            row["stream_copies"] = copies
+            row["frac_of_hbm_stream"] = round(compulsory_bytes(c.g) / (t_stream * 1e-3) / 1e9 / hbm_peak, 4)
         if i in read_ms:
             row["read_ceiling_ms"] = round(read_ms[i], 5)
             row["frac_of_read_ceiling"] = round(read_ms[i] / ms, 4)
@@ -746,8 +797,29 @@ def run_sweep(args, dev):
             "wall_s": round(wall, 1), "points_file": args.sweep}
 
 
+def parse_shape(text: str) -> W.Gemm:
+    """One GEMM from 'DTYPE:MxNxK:LAYOUT', e.g. 'int8:5120x5120x5120:row'
+    (DTYPE int8, int8_int16, int8_int8 or bf16; LAYOUT row or col): int8
+    operands uniform on [-128, 127], bf16 N(0, 1), seed 0, shift 7 for the
+    requantised outputs."""
+    try:
+        dtype, dims, lay = text.split(":")
+        M, N, K = (int(x) for x in dims.lower().split("x"))
+    except ValueError:
+        raise SystemExit(f"--shape wants DTYPE:MxNxK:LAYOUT, got {text!r}")
+    if dtype not in ("int8", "int8_int16", "int8_int8", "bf16") or lay not in ("row", "col") or min(M, N, K) < 1:
+        raise SystemExit(f"--shape: unknown dtype / layout or empty size in {text!r}")
+    d = W.BF if dtype == "bf16" else W.I8
+    return W.Gemm(M, N, K, dtype, W.B_ROW_MAJOR if lay == "row" else W.B_COL_MAJOR, 0, d, d,
+                  7 if dtype in ("int8_int16", "int8_int8") else 0)
+
+
 def select(args) -> W.Workload:
-    """The workload, optionally narrowed to the GEMMs named by --gemm."""
+    """The workload (or the one GEMM of --shape), optionally narrowed to the
+    GEMMs named by --gemm."""
+    if args.shape:
+        g = parse_shape(args.shape)
+        return W.Workload("shape", f"one GEMM {g.name}, seed 0", (g,))
     wl = W.WORKLOADS[args.workload]
     if not args.gemm:
         return wl
@@ -764,10 +836,13 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="all_configs", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--shape", metavar="DTYPE:MxNxK:LAYOUT",
+                    help="time one GEMM of this shape instead of a workload, e.g. int8:5120x5120x5120:row")
     ap.add_argument("--gemm", action="append", default=[],
                     help="run only this GEMM of the workload (repeatable), e.g. bf16_4096x4096x4096_Bcol")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-stream", action="store_true", help="skip the back-to-back pass of the HBM-bound GEMMs")
     ap.add_argument("--cpu-seconds", type=float, default=30.0)
     ap.add_argument("--cpu-seconds-per-step", type=float, default=6.0)
     ap.add_argument("--sweep", metavar="OUT.json",

@@ -226,7 +226,9 @@ gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream
  *   out->route: GEMM_ROUTE_*; bn: tile width (the small operand's tile
  *   height for GEMM_ROUTE_SMALL_OPERAND); splits: K split factor; stages:
  *   pipeline depth of the tensor-core kernel; grid: CTAs launched;
- *   model_us: modelled time of the tensor-core kernel and split-K reduction.
+ *   model_us: modelled time of the tensor-core kernel and split-K reduction
+ *   (the quantity the planner minimises); dram_us: the DRAM time of the
+ *   model's traffic at the copy bandwidth (above model_us: memory-bound).
  * Returns GEMM_ERR_INVALID_ARG / GEMM_ERR_UNSUPPORTED like the GEMM calls.
  */
 enum {
@@ -245,6 +247,7 @@ typedef struct {
   int stages;
   int grid;
   double model_us;
+  double dram_us;
 } gemm_plan_t;
 gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_layout, int sms, int pair_slots,
                               gemm_plan_t *out);

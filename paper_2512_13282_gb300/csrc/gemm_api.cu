@@ -252,31 +252,36 @@ struct Plan {
 // tile, BN among the compiled widths, K split S ways -- runs in
 // ceil(tiles * S / slots) rounds of one unit per slot (an SM or an SM pair);
 // its modelled time is
-//   max(rounds * (kb_per_unit * kstep + unit), DRAM time) + split terms
-// (Eq. 9 with wave quantisation, Eq. 6-8 and 10), with the per-variant K-step
-// and unit costs and the split constants fitted to measurements on GB300
-// (plan_table.h, generated by tile_model.py).  The least time wins; on a tie
-// the earlier candidate (single CTA before pair, wider before narrower,
-// fewer splits before more).  tile_model.choose_plan is the same rule.
-double modelled_us(int64_t M, int64_t N, int64_t K, bool int8, bool pair, int bn, int64_t splits, int64_t kb_per,
+//   rounds * (kb_per_unit * kstep + unit) + split terms
+// (Eq. 9 with wave quantisation), with the per-variant K-step and unit costs
+// and the split constants fitted to measurements on GB300 (plan_table.h,
+// generated by tile_model.py).  The least time wins; on a tie the earlier
+// candidate (single CTA before pair, wider before narrower, fewer splits
+// before more).  tile_model.choose_plan is the same rule.  The DRAM time of
+// Eq. 6-8 and 10 (dram_us) classifies the GEMM but does not rank plans: with
+// the 129 MB L2 supplying the reuse, it barely depends on the tile.
+double modelled_us(int64_t M, int64_t N, bool int8, bool pair, int bn, int64_t splits, int64_t kb_per,
                    int64_t rounds) {
   const int wi = bn == 128 ? 0 : bn == 192 ? 1 : bn == 224 ? 2 : 3;
   const plan_table::StepCost c = plan_table::kCost[int8 ? 1 : 0][pair ? 1 : 0][wi];
-  const double t_comp = (double)rounds * ((double)kb_per * c.kstep_us + c.unit_us);
-  // DRAM bytes: operands (bf16 in the kernel), re-reads of B when neither B
-  // nor both operands stay in L2, C, split-K partials written and read
-  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * K * N;
-  double rb = 1.0;
-  if (!(b_bytes <= plan_table::kL2Bytes / 2 || a_bytes + b_bytes <= plan_table::kL2Bytes)) {
-    rb = (double)ceil_div(M, kBM) / 8.0;
-    if (rb < 1.0) rb = 1.0;
-  }
-  const double c_bytes = (double)M * N * (int8 ? 4 : 2) + (splits > 1 ? 8.0 * splits * M * N : 0.0);
-  const double t_mem = (a_bytes + b_bytes * rb + c_bytes) / (plan_table::kHbmGBs * 1e3);
-  double t = t_comp > t_mem ? t_comp : t_mem;
+  double t = (double)rounds * ((double)kb_per * c.kstep_us + c.unit_us);
   if (splits > 1)
     t += plan_table::kSplitFixedUs[int8 ? 1 : 0] + plan_table::kSplitUsPerMB[int8 ? 1 : 0] * 4.0 * splits * M * N / 1e6;
   return t;
+}
+
+// Eq. 6-8 and 10: DRAM bytes of A (once: the grouped raster keeps a group's
+// 8 row tiles of A in L2 while it sweeps N), B (once if it, or A and B
+// together, fit in L2, else once per group of 8 row tiles) and C, at the
+// copy bandwidth, in microseconds.
+double dram_us(int64_t M, int64_t N, int64_t K, bool int8, bool pair) {
+  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * K * N;
+  double rb = 1.0;
+  if (!(b_bytes <= plan_table::kL2Bytes / 2 || a_bytes + b_bytes <= plan_table::kL2Bytes)) {
+    rb = (double)ceil_div(M, 8 * (pair ? 2 * kBM : kBM));
+    if (rb < 1.0) rb = 1.0;
+  }
+  return (a_bytes + b_bytes * rb + (double)M * N * (int8 ? 4 : 2)) / (plan_table::kHbmGBs * 1e3);
 }
 
 Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms, int pairs) {
@@ -321,7 +326,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
           if (s2 > 1 && (kb_per < 4 || tiles * s2 > 2 * slots)) continue;
         }
         seen[nseen++] = s2;
-        const double cost = modelled_us(M, N, K, int8, pair, bn, s2, kb_per, ceil_div(tiles * s2, slots));
+        const double cost = modelled_us(M, N, int8, pair, bn, s2, kb_per, ceil_div(tiles * s2, slots));
         if (best_cost < 0 || cost < best_cost - 1e-9) {
           best_cost = cost;
           best_pair = pair;
@@ -901,6 +906,7 @@ gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_l
   out->stages = tc_max_stages(pl.v.pair ? pl.v.bn / 2 : pl.v.bn, ew, pl.v.tma_out);
   out->grid = pl.grid;
   out->model_us = pl.model_us;
+  out->dram_us = dram_us(M, N, K, int8 != 0, pl.v.pair);
   return GEMM_OK;
 }
 

@@ -42,8 +42,11 @@ pipeline stage, accumulating in TMEM.  The restatement:
   Split-K, which the paper never uses, adds the partials' traffic and a
   reduction launch: T_split = r0 + r1 * (4 * S * M * N bytes).
 
-The planner (csrc/gemm_api.cu make_plan) minimises max(T_comp, T_mem) +
-T_split over (family, BN, S) with the per-variant t_kstep and t_unit and the
+With the 129 MB L2 supplying the reuse, T_mem hardly depends on the tile
+(unlike the NPU's, where m_ct and n_ct set the DRAM traffic directly), so it
+classifies a GEMM (compute- or memory-bound, the paper's balance) but does
+not rank plans.  The planner (csrc/gemm_api.cu make_plan) minimises
+T_comp + T_split over (family, BN, S) with the per-variant t_kstep and t_unit and the
 split constants that fit() derives from measurements (tile_sweep.py) and
 header_text() writes to csrc/plan_table.h.  balanced_search() is the paper's
 iterative procedure on the same candidates: the model proposes, measurements
@@ -211,20 +214,26 @@ def candidate_plans(M, N, K, b_kmajor, sms=None, pair_slots=None):
 # ------------------------------------------------------------------ cost
 
 def mem_time_us(M, N, K, dtype, plan):
-    """Eq. 6-8 and 10 for one plan, in microseconds."""
+    """Eq. 6-8 and 10 for one plan, in microseconds: A once (the grouped
+    raster keeps a group's 8 row tiles of A in L2 while it sweeps N), B once
+    if it (or A and B together) fits in L2, else once per group of 8 row
+    tiles (128 or 256 rows each: CTA pairs halve the re-reads), C once.
+    Split-K partials are left out: they stay in L2, and their cost is the
+    fitted split term."""
     ty = 2  # operands are bf16 in the kernel (int8 is staged as bf16)
     tyc = 4 if dtype == "int8" else 2
     l2 = GB300["l2_bytes"]
     a_bytes, b_bytes = M * K * ty, K * N * ty
-    ra = 1.0
-    rb = 1.0 if (b_bytes <= l2 / 2 or a_bytes + b_bytes <= l2) else max(1.0, _ceil(M, BM) / 8)
-    c_bytes = M * N * tyc + (2 * 4 * plan["splits"] * M * N if plan["splits"] > 1 else 0)
-    return (a_bytes * ra + b_bytes * rb + c_bytes) / (GB300["hbm_gbs"] * 1e3)
+    rows_per_group = 8 * (2 * BM if plan["pair"] else BM)
+    rb = 1.0 if (b_bytes <= l2 / 2 or a_bytes + b_bytes <= l2) else max(1.0, float(_ceil(M, rows_per_group)))
+    return (a_bytes + b_bytes * rb + M * N * tyc) / (GB300["hbm_gbs"] * 1e3)
 
 
 def plan_cost_us(M, N, K, dtype, plan, table):
-    """max(T_comp, T_mem) + T_split (Eq. 9, 10 and the split term) with the
-    fitted per-variant costs of `table`."""
+    """T_comp + T_split (Eq. 9 with wave quantisation, and the split term)
+    with the fitted per-variant costs of `table`: the time the planner
+    minimises.  Eq. 10's DRAM time (mem_time_us) is reported beside it; with
+    a 129 MB L2 it barely depends on the plan, so it does not rank plans."""
     g = table["groups"].get(group_key(dtype, plan["pair"], plan["bn"]))
     if g is None:
         return math.inf
@@ -233,7 +242,7 @@ def plan_cost_us(M, N, K, dtype, plan, table):
     if plan["splits"] > 1:
         sp = table["split"][dtype]
         t_split = sp["fixed_us"] + sp["us_per_mb"] * 4 * plan["splits"] * M * N / 1e6
-    return max(t_comp, mem_time_us(M, N, K, dtype, plan)) + t_split
+    return t_comp + t_split
 
 
 def group_key(dtype, pair, bn):

@@ -52,3 +52,13 @@ def test_recorded_traffic_families_are_known(fam):
     for e in rec["dram_bytes_per_launch"].values():
         assert e["family"] in bench.KERNEL_FAMILIES
         assert e["bytes"] > 0
+
+
+def test_parse_shape():
+    g = bench.parse_shape("int8:5120x4096x3000:row")
+    assert (g.M, g.N, g.K, g.dtype, g.layout) == (5120, 4096, 3000, "int8", 0)
+    g = bench.parse_shape("bf16:1x2x3:col")
+    assert g.dtype == "bf16" and g.layout == 1
+    for bad in ("int4:1x1x1:row", "int8:1x1:row", "int8:1x1x1:diag", "int8:0x1x1:row"):
+        with pytest.raises(SystemExit):
+            bench.parse_shape(bad)

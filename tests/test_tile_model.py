@@ -104,6 +104,7 @@ def test_library_planner_equals_the_model(lib):
         got = (plan["route"] == G.GEMM_ROUTE_TC_PAIR, plan["bn"], plan["splits"])
         assert got == (want["pair"], want["bn"], want["splits"]), (M, N, K, dtype, layout, plan, want)
         assert plan["model_us"] == pytest.approx(T.plan_cost_us(M, N, K, dtype, want, table), rel=1e-4)
+        assert plan["dram_us"] == pytest.approx(T.mem_time_us(M, N, K, dtype, want), rel=1e-6)
         checked += 1
     assert checked > 150
 
