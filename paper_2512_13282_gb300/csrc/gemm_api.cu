@@ -491,9 +491,8 @@ gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const 
                          const void *B, int64_t ldb, bool b_kmajor, void *C, int64_t ldc, bool int8,
                          cudaStream_t st, int out_bits = 32, int out_shift = 0) {
   const bool row_b = !b_kmajor;
-  const int64_t strips = ceil_div(N, row_b ? 256 : 32);
   SkinnyParams p{};
-  skinny_split(K, strips, d.sms, (int)M, int8 ? 1 : 2, &p.kb, &p.ks);
+  const int64_t strips = skinny_geometry((int)M, N, K, int8, row_b, d.sms, &p.kb, &p.ks);
   p.A = A;
   p.lda = lda;
   p.B = B;
@@ -506,11 +505,8 @@ gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const 
   p.out_bits = out_bits;
   p.out_shift = out_shift;
   const int esize = int8 ? 1 : 2;
-  const uintptr_t bb = reinterpret_cast<uintptr_t>(B);
-  if (row_b && int8)
-    p.b_vec = (bb % 8 == 0) && (ldb % 8 == 0);
-  else
-    p.b_vec = (bb % 16 == 0) && ((ldb * esize) % 16 == 0);
+  const uint64_t bits = reinterpret_cast<uintptr_t>(B) | (uint64_t)(ldb * esize) | 16u;
+  p.b_align = (int)(bits & (~bits + 1));  // lowest set bit: 1, 2, 4, 8 or 16
   gemm_status_t s;
   if (p.ks > 1) {
     if ((s = ensure_workspace(d, (size_t)p.ks * M * N * 4, st)) != GEMM_OK) return s;
@@ -521,7 +517,7 @@ gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const 
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
   g_launches.fetch_add(1);
-  if (launch_skinny(p, int8, row_b, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (launch_skinny(p, int8, row_b, strips, st) != cudaSuccess) return GEMM_ERR_CUDA;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
   return GEMM_OK;
 }

@@ -183,15 +183,16 @@ struct SkinnyParams {
   int64_t ldc;
   int M;
   int64_t N, K;
-  int kb;              // rows of K per block slice (multiple of 32)
+  int kb;              // rows of K per block slice (skinny_geometry)
   int ks;              // slices (blocks per column strip)
-  int b_vec;           // B rows allow 16-byte (8-byte for row-major int8) loads
+  int b_align;         // 16, 8, 4, 2 or 1: alignment in bytes of the B base and row pitch
   void *ws;            // ks x M x N 32-bit partials (ks > 1)
   uint32_t *tickets;   // one zeroed counter per column strip (ks > 1)
   int out_bits;        // int8: 32 (int32 C), 16 or 8 (requantised C)
   int out_shift;       // int8 with out_bits < 32: right shift, 0..31
 };
-void skinny_split(int64_t K, int64_t strips, int sms, int m_rows, int esize, int *kb, int *ks);
-cudaError_t launch_skinny(const SkinnyParams &p, bool int8, bool row_b, cudaStream_t st);
+// Column strips of the launch (the grid's x); fills kb and ks.
+int64_t skinny_geometry(int M, int64_t N, int64_t K, bool int8, bool row_b, int sms, int *kb, int *ks);
+cudaError_t launch_skinny(const SkinnyParams &p, bool int8, bool row_b, int64_t strips, cudaStream_t st);
 
 }  // namespace gb300

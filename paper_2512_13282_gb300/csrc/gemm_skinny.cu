@@ -4,21 +4,25 @@
 // every element of B is used M times, far too few for the tensor cores to
 // matter, and the time is the time to stream B from HBM once (the paper
 // lists GEMV as future work, Sec. 5.3.4).  This kernel streams B with
-// 16-byte coalesced loads and keeps A in shared memory:
+// coalesced loads, many in flight per lane, and keeps A in shared memory:
 //
-//   - B row-major (K x N): a lane owns 8 consecutive columns and walks rows
-//     k; a warp reads 256 contiguous bf16 (or 32 lanes x 8 int8) per row.
+//   - B row-major (K x N): a lane owns 4, 8 or 16 contiguous bytes of columns
+//     and walks rows k; a warp reads 128-512 contiguous bytes per row.  The
+//     lane width, the bytes a lane has in flight and the blocks per SM
+//     depend on M and the type (rowb_shape), and the grid is one wave.
 //   - B column-major (N x K): a warp owns 4 columns (rows of the storage)
 //     and its lanes split K in 16-byte chunks; partial dot products are
 //     summed across lanes at the end.
 //   - int8 uses __dp4a (4 exact int8 products summed into int32); a row-major
-//     B chunk of 4 rows x 8 columns is byte-transposed so that each word holds
+//     B piece of 4 rows x 4 columns is byte-transposed so that each word holds
 //     4 consecutive k of one column.  bf16 accumulates in fp32 FMAs.
 //   - K is split across the 8 warps of a block and across `ks` blocks per
 //     column strip; the last block of a strip to finish (atomic ticket) adds
 //     the fp32/int32 partials of all blocks in a fixed order, so results do
 //     not depend on scheduling, and rounds once to bf16.
 #include <cuda_bf16.h>
+
+#include <type_traits>
 
 #include "gemm_internal.h"
 
@@ -88,13 +92,28 @@ __device__ void finish_block(const SkinnyParams &p, const uint32_t *vals, int ld
   for (int t = threadIdx.x; t < total; t += kSkThreads) {
     const int m = t / cols, c = t - m * cols;
     const int64_t n = n0 + c;
+    // slices 0, 1, ... in order, four loads in flight at a time
+    uint32_t v[4];
+    int k = 0;
     if (INT8) {
       int32_t s = 0;
-      for (int k = 0; k < p.ks; ++k) s += (int32_t)__ldcg(partial_ptr(p, k, m, n));
+      for (; k + 4 <= p.ks; k += 4) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __ldcg(partial_ptr(p, k + i, m, n));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) s += (int32_t)v[i];
+      }
+      for (; k < p.ks; ++k) s += (int32_t)__ldcg(partial_ptr(p, k, m, n));
       store_s8_out(p, m, n, s);
     } else {
       float s = 0.f;
-      for (int k = 0; k < p.ks; ++k) s += __uint_as_float(__ldcg(partial_ptr(p, k, m, n)));
+      for (; k + 4 <= p.ks; k += 4) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __ldcg(partial_ptr(p, k + i, m, n));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) s += __uint_as_float(v[i]);
+      }
+      for (; k < p.ks; ++k) s += __uint_as_float(__ldcg(partial_ptr(p, k, m, n)));
       __nv_bfloat16 h = __float2bfloat16_rn(s);
       reinterpret_cast<uint16_t *>(p.C)[m * p.ldc + n] = *reinterpret_cast<uint16_t *>(&h);
     }
@@ -103,178 +122,214 @@ __device__ void finish_block(const SkinnyParams &p, const uint32_t *vals, int ld
 }
 
 // ------------------------------------------------------------ B row-major
-// Block = 256 columns (8 per lane) x a K range; warp w takes rows
-// k0 + w, k0 + w + 8, ... of the range.  MT = rows of A held (>= M).
-template <int MT, bool INT8>
-__global__ void __launch_bounds__(kSkThreads) skinny_rowB_kernel(const SkinnyParams p) {
-  constexpr int kCols = 256;
+// A lane owns VB contiguous bytes of every row it reads (VB / esize columns)
+// and a warp 32 * VB bytes: the block's column strip.  The block's K slice is
+// cut into batches of R = RB / VB rows; warp w takes batches w, w + 8, ...
+// Each batch is loaded in two halves, and a half is reloaded with the next
+// batch's rows as soon as it has been multiplied, so every lane keeps RB / 2
+// to RB bytes of B in flight.  The first loads are issued before A is staged
+// in shared memory.  int8 byte-transposes each 4-row x 4-column piece so that
+// a word holds four k of one column for __dp4a.
+constexpr int mt_of(int M) { return M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16; }
+
+// Launch shape of the row-major kernel per rows of A held (MT) and type:
+// bytes of a B row a lane loads (VB), bytes a lane loads per batch (RB) and
+// resident blocks per SM (BPS, which caps the registers a thread at 64, 80
+// or 128).  Chosen on GB300 by timing every (VB, RB, BPS) on M = 1, 4, 8, 16
+// with N = 4096..11008, K = 4096: narrower lanes with more blocks win for
+// int8 (8-byte lanes, 16 KB of B in flight per block, 4 blocks per SM at
+// M = 1; 4-byte lanes, 8 KB per block, at M = 8), wider lanes for bf16,
+// whose fp32 accumulators leave fewer registers.
+struct RowBShape {
+  int vb, rb, bps;
+};
+constexpr RowBShape rowb_shape(int mt, bool int8) {
+  return int8 ? (mt == 1 ? RowBShape{8, 128, 4} : mt == 2 ? RowBShape{8, 128, 3} : mt == 4 ? RowBShape{8, 128, 2}
+                 : RowBShape{4, 64, mt == 8 ? 3 : 2})
+              : (mt == 1 ? RowBShape{8, 128, 4} : mt == 2 ? RowBShape{8, 128, 3} : mt <= 8 ? RowBShape{8, 128, 2}
+                 : RowBShape{4, 128, 2});
+}
+
+template <int MT, int VB, bool INT8, int RB, int BPS>
+__global__ void __launch_bounds__(kSkThreads, BPS) skinny_rowB_kernel(const SkinnyParams p) {
+  constexpr int R = RB / VB;              // rows per batch
+  constexpr int H = R / 2;                // rows per half batch (a multiple of 4)
+  static_assert(H >= 1 && (!INT8 || H % 4 == 0), "int8 half batches are whole quads of rows");
+  constexpr int W = VB / 4;               // 32-bit words per lane per row
+  constexpr int CPL = INT8 ? VB : VB / 2; // columns per lane
+  constexpr int kCols = 32 * CPL;         // columns per block
+  constexpr int esize = INT8 ? 1 : 2;
   extern __shared__ uint32_t sk_smem[];
-  uint32_t *a_s = sk_smem;                        // A slice: MT x kb (bf16 as fp32 bits, or int8 words)
   __shared__ uint32_t ticket;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n0 = (int64_t)blockIdx.x * kCols;
   const int64_t k0 = (int64_t)blockIdx.y * p.kb;
-  const int kb = (int)min((int64_t)p.kb, (int64_t)p.K - k0);  // rows of this slice (> 0)
-  // stage A[0:M, k0:k0+kb] (zero for m >= M)
-  if (INT8) {
-    const int words = (kb + 3) / 4;
+  const int kb = (int)min((int64_t)p.kb, p.K - k0);  // rows of this slice (> 0)
+  const int batches = (kb + R - 1) / R;
+  const int64_t col = n0 + lane * CPL;
+  const bool vec = p.b_align >= VB && col + CPL <= p.N;
+  const uint8_t *Bb = reinterpret_cast<const uint8_t *>(p.B) + (k0 * p.ldb + col) * esize;
+  const int64_t pitch = p.ldb * esize;
+
+  // rows [r0, r0 + H) of the slice into w (zero past the slice and past N)
+  auto load_half = [&](int r0, uint32_t (&w)[H][W]) {
+#pragma unroll
+    for (int r = 0; r < H; ++r) {
+#pragma unroll
+      for (int j = 0; j < W; ++j) w[r][j] = 0u;
+      if (r0 + r >= kb) continue;
+      const uint8_t *row = Bb + (int64_t)(r0 + r) * pitch;
+      if (vec) {
+        if constexpr (VB == 16) {
+          const uint4 v = __ldcs(reinterpret_cast<const uint4 *>(row));
+          w[r][0] = v.x; w[r][1] = v.y; w[r][2] = v.z; w[r][3] = v.w;
+        } else if constexpr (VB == 8) {
+          const uint2 v = __ldcs(reinterpret_cast<const uint2 *>(row));
+          w[r][0] = v.x; w[r][1] = v.y;
+        } else {
+          w[r][0] = __ldcs(reinterpret_cast<const unsigned int *>(row));
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < CPL; ++c)
+          if (col + c < p.N) {
+            const uint32_t v = INT8 ? (uint32_t)row[c] : (uint32_t)reinterpret_cast<const uint16_t *>(row)[c];
+            w[(r)][(c * esize) >> 2] |= v << (8 * ((c * esize) & 3));
+          }
+      }
+    }
+  };
+
+  uint32_t h0[H][W], h1[H][W];
+  int b = warp;
+  load_half(b * R, h0);
+  load_half(b * R + H, h1);
+
+  // stage A[0:M, k0:k0+kb] (zero for m >= M and past the slice, up to whole
+  // batches): int8 as words of 4 k, bf16 as fp32
+  const int kbp = batches * R;
+  const int words = kbp / 4;
+  uint32_t *a_s = sk_smem;
+  if constexpr (INT8) {
     for (int t = threadIdx.x; t < MT * words; t += kSkThreads) {
-      const int m = t / words, w = t - m * words;
+      const int m = t / words, q = t - m * words;
       uint32_t v = 0;
       if (m < p.M) {
-        const int8_t *a = reinterpret_cast<const int8_t *>(p.A) + (int64_t)m * p.lda + k0 + 4 * w;
+        const int8_t *a = reinterpret_cast<const int8_t *>(p.A) + (int64_t)m * p.lda + k0 + 4 * q;
         for (int i = 0; i < 4; ++i)
-          if (4 * w + i < kb) v |= (uint32_t)(uint8_t)a[i] << (8 * i);
+          if (4 * q + i < kb) v |= (uint32_t)(uint8_t)a[i] << (8 * i);
       }
-      a_s[m * words + w] = v;
+      a_s[t] = v;
     }
   } else {
-    for (int t = threadIdx.x; t < MT * kb; t += kSkThreads) {
-      const int m = t / kb, k = t - m * kb;
+    for (int t = threadIdx.x; t < MT * kbp; t += kSkThreads) {
+      const int m = t / kbp, k = t - m * kbp;
       float v = 0.f;
-      if (m < p.M) v = __uint_as_float((uint32_t)reinterpret_cast<const uint16_t *>(p.A)[(int64_t)m * p.lda + k0 + k] << 16);
-      a_s[m * kb + k] = __float_as_uint(v);
+      if (m < p.M && k < kb)
+        v = __uint_as_float((uint32_t)reinterpret_cast<const uint16_t *>(p.A)[(int64_t)m * p.lda + k0 + k] << 16);
+      a_s[t] = __float_as_uint(v);
     }
   }
   __syncthreads();
 
-  const int64_t col = n0 + lane * 8;
-  const bool vec = col + 8 <= p.N && p.b_vec;
-  if (INT8) {
-    int32_t acc[MT][8];
+  using Acc = typename std::conditional<INT8, int32_t, float>::type;
+  Acc acc[MT][CPL];
 #pragma unroll
-    for (int m = 0; m < MT; ++m)
+  for (int m = 0; m < MT; ++m)
 #pragma unroll
-      for (int c = 0; c < 8; ++c) acc[m][c] = 0;
-    const int8_t *B = reinterpret_cast<const int8_t *>(p.B);
-    const int words = (kb + 3) / 4;
-    // warp w handles k-quads 2w, 2w+1, then +16, ...: 8 rows in flight
-    for (int qbase = 2 * warp; qbase < words; qbase += 2 * kSkWarps) {
-      uint32_t lo[2][4], hi[2][4];  // 8 columns of 4 rows, two quads
+    for (int c = 0; c < CPL; ++c) acc[m][c] = 0;
+
+  // multiply rows [r0, r0 + H) held in w
+  auto mul_half = [&](int r0, const uint32_t (&w)[H][W]) {
+    if constexpr (INT8) {
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
+      for (int q = 0; q < H / 4; ++q) {
+        const int aq = (r0 >> 2) + q;  // A word of these four rows
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          lo[h][i] = hi[h][i] = 0;
-          const int kq = 4 * (qbase + h) + i;
-          if (kq >= kb) continue;
-          const int8_t *row = B + (k0 + kq) * p.ldb + col;
-          if (vec) {
-            const uint2 v = __ldcs(reinterpret_cast<const uint2 *>(row));
-            lo[h][i] = v.x;
-            hi[h][i] = v.y;
-          } else {
-            for (int c = 0; c < 8; ++c)
-              if (col + c < p.N) {
-                const uint32_t b = (uint8_t)row[c];
-                if (c < 4) lo[h][i] |= b << (8 * c); else hi[h][i] |= b << (8 * (c - 4));
-              }
+        for (int j = 0; j < W; ++j) {
+          const uint32_t x0 = w[4 * q][j], x1 = w[4 * q + 1][j], x2 = w[4 * q + 2][j], x3 = w[4 * q + 3][j];
+          const uint32_t lo01 = __byte_perm(x0, x1, 0x5140), hi01 = __byte_perm(x0, x1, 0x7362);
+          const uint32_t lo23 = __byte_perm(x2, x3, 0x5140), hi23 = __byte_perm(x2, x3, 0x7362);
+          const uint32_t cw[4] = {__byte_perm(lo01, lo23, 0x5410), __byte_perm(lo01, lo23, 0x7632),
+                                  __byte_perm(hi01, hi23, 0x5410), __byte_perm(hi01, hi23, 0x7632)};
+#pragma unroll
+          for (int m = 0; m < MT; ++m) {
+            const int aw = (int)a_s[m * words + aq];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+              acc[m][4 * j + c] = __dp4a(aw, (int)cw[c], acc[m][4 * j + c]);
           }
         }
+      }
+    } else {
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int q = qbase + h;
-        if (q >= words) break;
-        // byte transpose: column word c = bytes c of rows 0..3
-        uint32_t cw[8];
+      for (int r = 0; r < H; ++r) {
+        float bv[CPL];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          // bytes [x.c, y.c] of two rows, then [r0.c, r1.c, r2.c, r3.c]
-          const uint32_t sel = (uint32_t)c | ((uint32_t)(c + 4) << 4);
-          const uint32_t s01 = __byte_perm(lo[h][0], lo[h][1], sel);
-          const uint32_t s23 = __byte_perm(lo[h][2], lo[h][3], sel);
-          cw[c] = __byte_perm(s01, s23, 0x5410);
-          const uint32_t t01 = __byte_perm(hi[h][0], hi[h][1], sel);
-          const uint32_t t23 = __byte_perm(hi[h][2], hi[h][3], sel);
-          cw[4 + c] = __byte_perm(t01, t23, 0x5410);
+        for (int j = 0; j < W; ++j) {
+          bv[2 * j] = bf16_lo(w[r][j]);
+          bv[2 * j + 1] = bf16_hi(w[r][j]);
         }
 #pragma unroll
         for (int m = 0; m < MT; ++m) {
-          const int aw = (int)a_s[m * words + q];
+          const float a = __uint_as_float(a_s[m * kbp + r0 + r]);
 #pragma unroll
-          for (int c = 0; c < 8; ++c) acc[m][c] = __dp4a(aw, (int)cw[c], acc[m][c]);
+          for (int c = 0; c < CPL; ++c) acc[m][c] = fmaf(a, bv[c], acc[m][c]);
         }
       }
     }
-    // combine the 8 warps in shared memory (reuse the A area after a sync)
-    __syncthreads();
-    uint32_t *red = sk_smem;  // MT x 256 words
+  };
+
+  for (; b < batches; b += kSkWarps) {
+    const int nb = b + kSkWarps;
+    if (b * R < kb) mul_half(b * R, h0);
+    if (nb < batches) load_half(nb * R, h0);
+    if (b * R + H < kb) mul_half(b * R + H, h1);
+    if (nb < batches) load_half(nb * R + H, h1);
+  }
+
+  // combine the 8 warps: int8 by shared-memory atomics (integer sums do not
+  // depend on order), bf16 through one slot per warp summed in warp order
+  __syncthreads();  // every warp is done with the A slice
+  uint32_t *red = sk_smem;
+  const int cols = (int)min((int64_t)kCols, p.N - n0);
+  if constexpr (INT8) {
     for (int t = threadIdx.x; t < MT * kCols; t += kSkThreads) red[t] = 0u;
     __syncthreads();
 #pragma unroll
     for (int m = 0; m < MT; ++m)
 #pragma unroll
-      for (int c = 0; c < 8; ++c) atomicAdd(reinterpret_cast<int *>(&red[m * kCols + lane * 8 + c]), acc[m][c]);
+      for (int c = 0; c < CPL; ++c) atomicAdd(reinterpret_cast<int *>(&red[m * kCols + lane * CPL + c]), (int)acc[m][c]);
     __syncthreads();
-    const int cols = (int)min((int64_t)kCols, (int64_t)p.N - n0);
     finish_block<true>(p, red, kCols, n0, cols, &ticket);
   } else {
-    float acc[MT][8];
+    float *slot = reinterpret_cast<float *>(sk_smem) + MT * kCols * warp;
 #pragma unroll
     for (int m = 0; m < MT; ++m)
 #pragma unroll
-      for (int c = 0; c < 8; ++c) acc[m][c] = 0.f;
-    const uint16_t *B = reinterpret_cast<const uint16_t *>(p.B);
-    constexpr int kRows = 4;  // rows in flight per lane
-    for (int kbase = warp * kRows; kbase < kb; kbase += kSkWarps * kRows) {
-      uint32_t w[kRows][4];
-#pragma unroll
-      for (int r = 0; r < kRows; ++r) {
-        w[r][0] = w[r][1] = w[r][2] = w[r][3] = 0;
-        const int k = kbase + r;
-        if (k >= kb) continue;
-        const uint16_t *row = B + (k0 + k) * p.ldb + col;
-        if (vec) {
-          const uint4 v = __ldcs(reinterpret_cast<const uint4 *>(row));
-          w[r][0] = v.x; w[r][1] = v.y; w[r][2] = v.z; w[r][3] = v.w;
-        } else {
-          for (int c = 0; c < 8; ++c)
-            if (col + c < p.N) w[r][c >> 1] |= (uint32_t)row[c] << (16 * (c & 1));
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < kRows; ++r) {
-        const int k = kbase + r;
-        if (k >= kb) break;
-        float b[8];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          b[2 * i] = bf16_lo(w[r][i]);
-          b[2 * i + 1] = bf16_hi(w[r][i]);
-        }
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-          const float a = __uint_as_float(a_s[m * kb + k]);
-#pragma unroll
-          for (int c = 0; c < 8; ++c) acc[m][c] = fmaf(a, b[c], acc[m][c]);
-        }
-      }
-    }
-    // combine the 8 warps in a fixed order (warp 0, 1, ...) in shared memory
+      for (int c = 0; c < CPL; ++c) slot[m * kCols + lane * CPL + c] = (float)acc[m][c];
     __syncthreads();
-    float *red = reinterpret_cast<float *>(sk_smem);  // MT x 256
-    for (int w2 = 0; w2 < kSkWarps; ++w2) {
-      if (warp == w2) {
+    float *sum = reinterpret_cast<float *>(sk_smem) + MT * kCols * kSkWarps;
+    for (int t = threadIdx.x; t < MT * kCols; t += kSkThreads) {
+      float s = 0.f;
 #pragma unroll
-        for (int m = 0; m < MT; ++m)
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            float &r = red[m * kCols + lane * 8 + c];
-            r = (w2 == 0) ? acc[m][c] : r + acc[m][c];
-          }
-      }
-      __syncthreads();
+      for (int w2 = 0; w2 < kSkWarps; ++w2) s += reinterpret_cast<const float *>(sk_smem)[MT * kCols * w2 + t];
+      sum[t] = s;
     }
-    const int cols = (int)min((int64_t)kCols, (int64_t)p.N - n0);
-    finish_block<false>(p, reinterpret_cast<uint32_t *>(red), kCols, n0, cols, &ticket);
+    __syncthreads();
+    finish_block<false>(p, reinterpret_cast<uint32_t *>(sum), kCols, n0, cols, &ticket);
   }
 }
 
 // --------------------------------------------------------- B column-major
 // Block = 32 columns (4 per warp) x a K range; lanes split the range in
 // 16-byte chunks of the B rows (the storage rows are the columns of B).
+// Resident blocks per SM of the column-major kernel, 5 down to 2 as its
+// registers grow with M (48 to 128 a thread).
+constexpr int colb_blocks(int mt) { return mt == 1 ? 5 : mt <= 4 ? 4 : mt == 8 ? 3 : 2; }
+
 template <int MT, bool INT8>
-__global__ void __launch_bounds__(kSkThreads) skinny_colB_kernel(const SkinnyParams p) {
+__global__ void __launch_bounds__(kSkThreads, colb_blocks(MT)) skinny_colB_kernel(const SkinnyParams p) {
   constexpr int kColsPerWarp = 4;
   constexpr int kCols = kColsPerWarp * kSkWarps;  // 32
   constexpr int kElems = INT8 ? 16 : 8;            // elements per 16-byte chunk
@@ -325,7 +380,7 @@ __global__ void __launch_bounds__(kSkThreads) skinny_colB_kernel(const SkinnyPar
       if (n >= p.N) continue;
       if (INT8) {
         const int8_t *row = reinterpret_cast<const int8_t *>(p.B) + n * p.ldb + k0 + kk;
-        if (p.b_vec && kk + kElems <= kb) {
+        if (p.b_align >= 16 && kk + kElems <= kb) {
           const uint4 v = __ldcs(reinterpret_cast<const uint4 *>(row));
           w[j][0] = v.x; w[j][1] = v.y; w[j][2] = v.z; w[j][3] = v.w;
         } else {
@@ -334,7 +389,7 @@ __global__ void __launch_bounds__(kSkThreads) skinny_colB_kernel(const SkinnyPar
         }
       } else {
         const uint16_t *row = reinterpret_cast<const uint16_t *>(p.B) + n * p.ldb + k0 + kk;
-        if (p.b_vec && kk + kElems <= kb) {
+        if (p.b_align >= 16 && kk + kElems <= kb) {
           const uint4 v = __ldcs(reinterpret_cast<const uint4 *>(row));
           w[j][0] = v.x; w[j][1] = v.y; w[j][2] = v.z; w[j][3] = v.w;
         } else {
@@ -392,10 +447,13 @@ __global__ void __launch_bounds__(kSkThreads) skinny_colB_kernel(const SkinnyPar
 template <int MT, bool INT8>
 cudaError_t launch_mt(const SkinnyParams &p, dim3 grid, bool row_b, cudaStream_t st) {
   if (row_b) {
-    const size_t a_bytes = INT8 ? (size_t)MT * ((p.kb + 3) / 4) * 4 : (size_t)MT * p.kb * 4;
-    const size_t red_bytes = (size_t)MT * 256 * 4;
+    constexpr RowBShape sh = rowb_shape(MT, INT8);
+    constexpr int VB = sh.vb;
+    constexpr int kCols = 32 * (INT8 ? VB : VB / 2);
+    const size_t a_bytes = INT8 ? (size_t)MT * p.kb : (size_t)MT * p.kb * 4;  // kb: whole batches
+    const size_t red_bytes = (size_t)MT * kCols * 4 * (INT8 ? 1 : kSkWarps + 1);
     const size_t smem = a_bytes > red_bytes ? a_bytes : red_bytes;
-    auto kern = skinny_rowB_kernel<MT, INT8>;
+    auto kern = skinny_rowB_kernel<MT, VB, INT8, sh.rb, sh.bps>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     kern<<<grid, kSkThreads, smem, st>>>(p);
@@ -414,29 +472,38 @@ cudaError_t launch_mt(const SkinnyParams &p, dim3 grid, bool row_b, cudaStream_t
 
 }  // namespace
 
-// Rows of K per block slice, and slices, for `strips` column strips: enough
-// blocks to cover the SMs a few times over, while the fp32/int32 partial
-// sums a slice writes (4 bytes per output) stay below 1/8 of the B bytes it
-// reads (kb >= 32 * m_rows / esize); slices are a multiple of 32 rows.
-void skinny_split(int64_t K, int64_t strips, int sms, int m_rows, int esize, int *kb, int *ks) {
-  const int64_t want_blocks = (int64_t)sms * 4;
-  int64_t s = (want_blocks + strips - 1) / strips;
-  const int64_t min_rows = (32 * (int64_t)m_rows + esize - 1) / esize;
-  const int64_t max_s = (K + (min_rows > 32 ? min_rows : 32) - 1) / (min_rows > 32 ? min_rows : 32);
+// Column strips, rows of K per block slice and slices.
+//  - Row-major B: one wave of blocks, as many slices as the resident blocks
+//    (rowb_shape) leave room for beside the column strips; slices are whole
+//    multiples of the block's 8 batches and hold at most 32 KB of A.
+//  - Column-major B: about four blocks per SM, slices a multiple of 32 rows,
+//    at most 2048.
+// Either way the fp32/int32 partial sums a slice writes (4 bytes per
+// output) stay below 1/8 of the B bytes it reads (kb >= 32 * M / esize).
+int64_t skinny_geometry(int M, int64_t N, int64_t K, bool int8, bool row_b, int sms, int *kb, int *ks) {
+  const int mt = mt_of(M), esize = int8 ? 1 : 2;
+  const RowBShape sh = rowb_shape(mt, int8);
+  const int64_t cols = row_b ? 32 * (sh.vb / esize) : 32;
+  const int64_t strips = (N + cols - 1) / cols;
+  const int64_t unit = row_b ? 8 * (sh.rb / sh.vb) : 32;
+  const int64_t max_rows = row_b ? (32768 / (mt * (int8 ? 1 : 4))) / unit * unit : 2048;
+  const int64_t min_rows = ((32 * (int64_t)(row_b ? mt : M) + esize - 1) / esize + unit - 1) / unit * unit;
+  int64_t s = row_b ? (int64_t)sms * sh.bps / strips                  // one wave
+                    : ((int64_t)sms * 4 + strips - 1) / strips;
+  const int64_t max_s = (K + min_rows - 1) / min_rows;
   if (s > max_s) s = max_s;
   if (s < 1) s = 1;
   int64_t rows = (K + s - 1) / s;
-  rows = (rows + 31) / 32 * 32;
-  if (rows > 2048) rows = 2048;  // bounds the A slice in shared memory
+  rows = (rows + unit - 1) / unit * unit;
+  if (rows > max_rows) rows = max_rows;
   *kb = (int)rows;
   *ks = (int)((K + rows - 1) / rows);
+  return strips;
 }
 
-cudaError_t launch_skinny(const SkinnyParams &p, bool int8, bool row_b, cudaStream_t st) {
-  const int64_t cols_per_block = row_b ? 256 : 32;
-  const dim3 grid((unsigned)((p.N + cols_per_block - 1) / cols_per_block), (unsigned)p.ks, 1);
-  const int mt = p.M <= 1 ? 1 : p.M <= 2 ? 2 : p.M <= 4 ? 4 : p.M <= 8 ? 8 : 16;
-  switch (mt) {
+cudaError_t launch_skinny(const SkinnyParams &p, bool int8, bool row_b, int64_t strips, cudaStream_t st) {
+  const dim3 grid((unsigned)strips, (unsigned)p.ks, 1);
+  switch (mt_of(p.M)) {
     case 1: return int8 ? launch_mt<1, true>(p, grid, row_b, st) : launch_mt<1, false>(p, grid, row_b, st);
     case 2: return int8 ? launch_mt<2, true>(p, grid, row_b, st) : launch_mt<2, false>(p, grid, row_b, st);
     case 4: return int8 ? launch_mt<4, true>(p, grid, row_b, st) : launch_mt<4, false>(p, grid, row_b, st);

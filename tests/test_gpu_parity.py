@@ -338,6 +338,29 @@ def test_small_m_misaligned_and_repeated(dtype, layout, monkeypatch):
         _check(dtype, A, B, layout, C)
 
 
+@pytest.mark.parametrize("dtype", ["int8", "bf16"])
+@pytest.mark.parametrize("M", [1, 2, 4, 8, 16])
+def test_small_m_row_b_alignments(dtype, M, monkeypatch):
+    """Row-major B whose base and row pitch are aligned to 16, 8, 4, 2 and 1
+    bytes: the small-M kernel loads 16, 8 or 4 bytes of a row per lane where
+    the alignment allows, else element by element; N ragged against every
+    lane width and K against the kernel's row batches."""
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "16")
+    esize = 1 if dtype == "int8" else 2
+    N, K = 1000, 1234
+    for align in (16, 8, 4, 2, 1):
+        if align < esize:
+            continue
+        el = align // esize  # elements of the alignment
+        ldb = -(-N // el) * el  # a pitch aligned to exactly `align` bytes (at least 16 for 16)
+        if align < 16 and (ldb * esize) % (2 * align) == 0:
+            ldb += el
+        b_off = 0 if align == 16 else el
+        A, B = _inputs(dtype, M, N, K, ROW, seed=align * 7 + M)
+        C = U.run(dtype, A, B, ROW, ldb=ldb, b_off=b_off)
+        _check(dtype, A, B, ROW, C)
+
+
 def test_small_m_int8_extremes(monkeypatch):
     """dp4a exactness at the int32 edge: K = 131071 of (-128)(-128)."""
     monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "16")
