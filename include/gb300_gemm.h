@@ -238,8 +238,7 @@ enum {
   GEMM_ROUTE_SMALL_OPERAND = 3,  /* int8 with one operand of <= 128 rows, converted in the kernel */
   GEMM_ROUTE_TC_SINGLE = 4,      /* tensor-core kernel, one CTA per 128 x BN tile */
   GEMM_ROUTE_TC_PAIR = 5,        /* tensor-core kernel, a CTA pair per 256 x BN tile */
-  GEMM_ROUTE_TINY = 6,           /* int8 problem small enough for one CUDA-core launch */
-  GEMM_ROUTE_TC_INT8_DIRECT = 7  /* int8 tensor-core kernel converting both operands inside (no staging) */
+  GEMM_ROUTE_TINY = 6            /* int8 problem small enough for one CUDA-core launch */
 };
 typedef struct {
   int route;

@@ -57,9 +57,7 @@ namespace {
 // plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
 // small-operand shapes, GB300_GEMM_TINY_MAX_MACS the largest
 // int8 problem (M * N * K) sent to the one-launch CUDA-core kernel (0
-// disables it), GB300_GEMM_S8X=0 / 1 the int8 kernel that converts both
-// operands inside never / wherever it is legal (-1, the default: where the
-// route rule picks it), GB300_GEMM_DEBUG=1 prints each plan.
+// disables it), GB300_GEMM_DEBUG=1 prints each plan.
 struct Overrides {
   int bn = 0;            // 0: planner's choice
   int pair = -1;         // -1: planner's choice
@@ -69,7 +67,6 @@ struct Overrides {
   bool pdl = true;
   bool s8tm = true;
   int64_t tiny_max_macs = -1;  // -1: built-in limit
-  int s8x = -1;          // -1: route rule; 0 never; 1 wherever legal
   bool debug = false;
 };
 
@@ -88,7 +85,6 @@ Overrides read_overrides() {
   o.pdl = env_int("GB300_GEMM_PDL", 1) != 0;
   o.s8tm = env_int("GB300_GEMM_S8TM", 1) != 0;
   if (const char *t = std::getenv("GB300_GEMM_TINY_MAX_MACS")) o.tiny_max_macs = std::atoll(t);
-  o.s8x = env_int("GB300_GEMM_S8X", -1);
   o.debug = env_int("GB300_GEMM_DEBUG", 0) != 0;
   return o;
 }
@@ -717,84 +713,6 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   return true;
 }
 
-// int8 operand of gemm_s8x_kernel, K contiguous: boxes of 64 bytes (k) x
-// box_rows rows, 64-byte swizzle (16-byte chunk j of row r at j ^ ((r / 2) % 4)).
-bool encode_s8_k64(CUtensorMap *map, const void *base, uint64_t K, uint64_t rows, uint64_t ld, uint32_t box_rows) {
-  const cuuint64_t dims[2] = {K, rows};
-  const cuuint64_t strides[1] = {ld};
-  const cuuint32_t box[2] = {64, box_rows};
-  const cuuint32_t estr[2] = {1, 1};
-  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// Whether the int8 GEMM takes gemm_s8x_kernel (both operands converted
-// inside, no staging).  Its TMA boxes need K-contiguous operands (B stored
-// N x K) with 16-byte aligned bases and pitches.
-bool s8x_legal(const void *A, int64_t lda, const void *B, int64_t ldb, bool b_kmajor) {
-  return b_kmajor && aligned16(A) && aligned16(B) && lda % 16 == 0 && ldb % 16 == 0;
-}
-
-bool s8x_chosen(int64_t M, int64_t N, int64_t K, bool legal) {
-  const int forced = overrides().s8x;
-  if (forced == 0 || !legal) return false;
-  if (forced == 1) return true;
-  (void)M;
-  (void)N;
-  (void)K;
-  return false;
-}
-
-bool try_s8x(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t lda, const int8_t *B,
-             int64_t ldb, bool b_kmajor, void *C, int64_t ldc, int out_bits, int shift, cudaStream_t st,
-             gemm_status_t *status) {
-  if (!s8x_chosen(M, N, K, s8x_legal(A, lda, B, ldb, b_kmajor))) return false;
-  TcParams p{};
-  p.M = (int)M;
-  p.N = (int)N;
-  p.K = (int)K;
-  p.tiles_m = (int)ceil_div(M, kBM);
-  p.tiles_n = (int)ceil_div(N, kS8xBN);
-  p.num_kb = (int)ceil_div(K, kBK);
-  p.splits = 1;
-  p.kb_per_split = p.num_kb;
-  p.slab_kb = 1024 / kBK;
-  p.group_m = 8;
-  p.out_bits = out_bits;
-  p.out_shift = shift;
-  const int out_esize = out_bits / 8;
-  const int64_t tiles = (int64_t)p.tiles_m * p.tiles_n;
-  const int grid = (int)(tiles < d.sms ? tiles : d.sms);
-  *status = GEMM_ERR_CUDA;
-  CUtensorMap ta, tb, tout;
-  if (!encode_s8_k64(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)lda, kBM)) return true;
-  if (!encode_s8_k64(&tb, B, (uint64_t)K, (uint64_t)N, (uint64_t)ldb, kS8xBN)) return true;
-  p.C = C;
-  p.ldc = ldc;
-  p.c_vec = aligned16(C) && ((ldc * out_esize) % 16 == 0);
-  p.ws = nullptr;
-  p.out_tma = kOutDirect;
-  tout = ta;
-  if (p.c_vec && overrides().tma_store) {
-    const CUtensorMapDataType type = out_bits == 32   ? CU_TENSOR_MAP_DATA_TYPE_INT32
-                                     : out_bits == 16 ? CU_TENSOR_MAP_DATA_TYPE_UINT16
-                                                      : CU_TENSOR_MAP_DATA_TYPE_UINT8;
-    if (!encode_out(&tout, type, (uint32_t)out_esize, C, (uint64_t)N, (uint64_t)M, (uint64_t)ldc, 1, 32))
-      return true;
-    p.out_tma = kOutTmaC;
-  }
-  p.err = d.err;
-  p.wait_limit_ns = wait_limit_ns();
-  const bool prof = g_prof_start && g_prof_stop;
-  if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
-  g_launches.fetch_add(1);
-  if (launch_s8x(ta, tb, tout, p, grid, st) != cudaSuccess) return true;
-  if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
-  *status = GEMM_OK;
-  return true;
-}
-
 // The int8 GEMM behind gemm_s8s8_s32 (out_bits 32), gemm_s8s8_s16 and
 // gemm_s8s8_s8 (out_bits 16 / 8, right shift `shift`): the exact int32 sum
 // is formed the same way for all three; only the final store differs.
@@ -827,7 +745,6 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
     return GEMM_OK;
   }
   if (try_s8tm(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, out_bits, shift, st, &s)) return s;
-  if (try_s8x(*d, M, N, K, A, lda, B, ldb, b_kmajor, C, ldc, out_bits, shift, st, &s)) return s;
   Plan pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms, pair_slots());
   pl.p.out_bits = out_bits;
   pl.p.out_shift = shift;
@@ -974,15 +891,6 @@ gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_l
     out->bn = qn;
     out->splits = (int)splits;
     out->grid = (int)(tiles * splits < sms ? tiles * splits : sms);
-    return GEMM_OK;
-  }
-  if (int8 && s8x_chosen(M, N, K, b_kmajor && K % 16 == 0)) {
-    const int64_t tiles = ceil_div(M, kBM) * ceil_div(N, kS8xBN);
-    out->route = GEMM_ROUTE_TC_INT8_DIRECT;
-    out->bn = kS8xBN;
-    out->splits = 1;
-    out->stages = kS8xStages;
-    out->grid = (int)(tiles < sms ? tiles : sms);
     return GEMM_OK;
   }
   const int epi = int8 ? kEpiS32 : kEpiBf16;

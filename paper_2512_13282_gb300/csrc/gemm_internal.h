@@ -113,17 +113,6 @@ cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64
 cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const S8tmParams &p, int grid,
                         cudaStream_t st);
 
-// int8 GEMM on the tensor cores with both operands converted to fp16 inside
-// the kernel (gemm_s8x.cu): A int8 M x K (K contiguous), B int8 N x K (K
-// contiguous), both 16-byte aligned with pitches a multiple of 16 bytes;
-// tiles of 128 x kS8xBN, no split-K (p.splits == 1); a: boxes of 64 k x 128
-// rows, b: 64 k x kS8xBN rows, 64-byte swizzle; o: C as for the general
-// int8 kernel (p.out_tma kOutTmaC or kOutDirect).
-constexpr int kS8xBN = 224;
-constexpr int kS8xStages = 4;  // int8 boxes in flight
-cudaError_t launch_s8x(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p, int grid,
-                       cudaStream_t st);
-
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
 // int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is
 // rows x cols with an arbitrary source leading dimension.

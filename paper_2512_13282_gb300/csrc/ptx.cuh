@@ -189,21 +189,6 @@ __device__ __forceinline__ void s8x4_to_bf16x4(uint32_t w, uint32_t &lo, uint32_
   hi = __byte_perm(f2, f3, 0x7632);
 }
 
-// Four int8 (byte i of w is element i) -> four fp16 bit patterns, elements
-// 0, 1 in lo and 2, 3 in hi (element 2i in the low half).  Byte b, flipped
-// to u = b + 128 in 0..255, is placed under the fp16 exponent of 1024: the
-// half 0x6400 | u is exactly 1024 + u (the unit in the last place of fp16 at
-// 1024 is 1).  One packed subtraction of 1152 = 1024 + 128 (0x6480) leaves
-// b, exactly (|b| <= 128 needs 8 significant bits; fp16 has 11).  Two byte
-// permutes and two packed subtractions for four elements.
-__device__ __forceinline__ void s8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
-  const uint32_t u = w ^ 0x80808080u;
-  const uint32_t bl = __byte_perm(u, 0x64646464u, 0x4140);  // halves 0x64:u0, 0x64:u1
-  const uint32_t bh = __byte_perm(u, 0x64646464u, 0x4342);  // halves 0x64:u2, 0x64:u3
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(lo) : "r"(bl), "r"(0x64806480u));
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(hi) : "r"(bh), "r"(0x64806480u));
-}
-
 // ----------------------------------------------------------------- tcgen05
 
 template <uint32_t kCols>
@@ -239,9 +224,8 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, ui
 }
 
 // D[tmem] (+)= A[tmem] * B[smem], kind::f16: A is 128 rows (TMEM lanes) of
-// K = 16 bf16 or fp16 (as the instruction descriptor says, the same type as
-// B) packed two to a 32-bit column (the lower k in the low half), i.e. 8
-// columns starting at a_tmem.
+// K = 16 bf16 packed two to a 32-bit column (the lower k in the low half),
+// i.e. 8 columns starting at a_tmem.
 __device__ __forceinline__ void tc_mma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
                                                    uint32_t idesc, uint32_t accumulate) {
   asm volatile(
@@ -267,11 +251,6 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
          ((n >> 3) << 17) | ((m >> 4) << 24);
-}
-
-// The same for fp16 A and B (formats 0), both K-major, fp32 D.
-__host__ __device__ constexpr uint32_t idesc_f16_f32(uint32_t m, uint32_t n) {
-  return (1u << 4) | ((n >> 3) << 17) | ((m >> 4) << 24);
 }
 
 // Shared-memory matrix descriptor, 128-byte swizzle:

@@ -35,7 +35,6 @@ GEMM_ROUTE_SMALL_OPERAND = 3
 GEMM_ROUTE_TC_SINGLE = 4
 GEMM_ROUTE_TC_PAIR = 5
 GEMM_ROUTE_TINY = 6
-GEMM_ROUTE_TC_INT8_DIRECT = 7
 
 
 class gemm_plan_t(ctypes.Structure):
