@@ -332,7 +332,7 @@ def run_ours(args, rank, world, dev):
             if k >= 2:
                 evs.append((a, b))
         torch.cuda.synchronize()
-        read_ms[i] = statistics.median(x.elapsed_time(y) for x, y in evs)
+        read_ms[i] = statistics.mean(x.elapsed_time(y) for x, y in evs)
         del buf
     # Back-to-back pass of the HBM-bound GEMMs (outside the timed steps):
     # R calls on R distinct operand copies whose bytes together exceed L2.
@@ -445,11 +445,16 @@ def run_ours(args, rank, world, dev):
 
     gemm_ms, e2e_max, wall = max_over_ranks([gemm_ms, e2e_ms or 0.0, wall], world, dev)
 
+    # Means over the steps: event-timed GEMMs of a few tens of microseconds
+    # right after the flush come out on a grid of about 2 us on GB300 (the
+    # events themselves resolve 32 ns), so a median lands on a grid point;
+    # the samples spread over neighbouring points, and their mean resolves
+    # the time between them.
     per = []
     for i, c in enumerate(cases):
-        ms = statistics.median(per_gemm_ms[i])
-        kms = statistics.median(per_kern_ms[i])
-        cms = statistics.median(per_clean_ms[i])
+        ms = statistics.mean(per_gemm_ms[i])
+        kms = statistics.mean(per_kern_ms[i])
+        cms = statistics.mean(per_clean_ms[i])
         tops = c.g.flops / (ms * 1e-3) / 1e12
         gbps = compulsory_bytes(c.g) / (ms * 1e-3) / 1e9
         row = {"gemm": c.g.name, "bound": bound_of(c.g, bf16_peak, hbm_peak), "ms": round(ms, 5),
@@ -687,7 +692,7 @@ def run_sweep(args, dev):
     each output precision and both B layouts.  Operands are the leading
     M*K / K*N elements of 8192^2 seeded master matrices (tight leading
     dimensions).  Each GEMM runs once untimed, then `reps` times, each after
-    an L2 flush, between CUDA events; the median is kept.  A few sampled
+    an L2 flush, between CUDA events; the mean is kept.  A few sampled
     entries of every result are checked against the oracle.  Writes every
     point to `args.sweep` (JSON) and returns the summary line."""
     import oracle
@@ -750,7 +755,7 @@ def run_sweep(args, dev):
                 r = np.concatenate([rng.integers(0, M, 3), [M - 1]])
                 c = np.concatenate([rng.integers(0, N, 3), [N - 1]])
                 got = C[torch.from_numpy(r).to(dev), torch.from_numpy(c).to(dev)].cpu().numpy()
-                ms = statistics.median(x.elapsed_time(y) for x, y in evs)
+                ms = statistics.mean(x.elapsed_time(y) for x, y in evs)
                 Ah = hA[:M * K].reshape(M, K)
                 Bh = hB[:K * N].reshape((K, N) if layout == W.B_ROW_MAJOR else (N, K))
                 if int8:
