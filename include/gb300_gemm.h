@@ -52,6 +52,10 @@
 #ifdef __cplusplus
 extern "C" {
 #endif
+/* The library is built with hidden symbols by default; these are its exports. */
+#if defined(__GNUC__)
+#pragma GCC visibility push(default)
+#endif
 
 typedef struct CUstream_st *gemm_stream_t; /* same object as cudaStream_t */
 
@@ -274,6 +278,9 @@ gemm_status_t gemm_selftest_read_stream(const void *ptr, size_t bytes, gemm_stre
  */
 void gemm_profile_events(void *start_event, void *stop_event);
 
+#if defined(__GNUC__)
+#pragma GCC visibility pop
+#endif
 #ifdef __cplusplus
 }
 #endif

@@ -20,7 +20,12 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_NAME = "libgb300gemm.so"
 LIB_PATH = os.path.join(HERE, LIB_NAME)
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
+# Internal symbols (kernel stubs, template instantiations) are hidden: a
+# process that loads another library defining the same names -- a second
+# copy of this one, say -- keeps each library's kernels its own.  The C ABI
+# is exported by the visibility pragma in gb300_gemm.h.
+NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
+              "-I" + INCLUDE, "-I" + CSRC]
 
 
 def _nvcc() -> str:

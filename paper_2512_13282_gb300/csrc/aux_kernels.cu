@@ -38,13 +38,27 @@ __device__ __forceinline__ void s8x16_to_bf16x16(const int4 raw, uint4 &lo, uint
 
 constexpr int kS8Threads = 256;
 
+// Row piece -> (row, first column) for pieces of `w` elements, `cpr` pieces
+// per row (32-bit division where the index allows it).
+__device__ __forceinline__ void piece_rc(uint64_t u, uint32_t cpr, int w, int64_t &r, int64_t &c) {
+  uint64_t rr, q;
+  if (u <= 0xFFFFFFFFull) {
+    rr = (uint32_t)u / cpr;
+    q = (uint32_t)u - (uint32_t)rr * cpr;
+  } else {
+    rr = u / cpr;
+    q = u - rr * cpr;
+  }
+  r = (int64_t)rr;
+  c = (int64_t)q * w;
+}
+
 // General path (any alignment, any leading dimension): both matrices as one
-// flat list of 4-element row pieces -- piece t < items_a is piece t % cpr_a
-// of row t / cpr_a of A (cpr = pieces per row), the rest likewise of B.
-// Consecutive threads take consecutive pieces of a row, so a warp reads 128
-// contiguous bytes (one 4-byte load per thread where the row allows it, four
-// byte loads otherwise) and writes 256 contiguous bytes (one 8-byte store:
-// staged rows start 16-byte aligned and pieces are 8 bytes apart).
+// flat list of 16-element row pieces -- piece t < items_a is piece t % cpr_a
+// of row t / cpr_a of A (cpr = pieces per row), the rest likewise of B.  A
+// thread reads its 16 bytes with the widest loads the row's address allows
+// (16, 8 or 4 bytes, else bytes), several in flight, and writes 32 bytes
+// with two 16-byte stores (staged rows start 16-byte aligned).
 __global__ void __launch_bounds__(kS8Threads)
     s8_to_bf16_pair_kernel(const S8Job a, const S8Job b, uint32_t cpr_a, uint32_t cpr_b, uint64_t items_a,
                            uint64_t items) {
@@ -53,30 +67,34 @@ __global__ void __launch_bounds__(kS8Threads)
   if (t >= items) return;
   const bool in_a = t < items_a;
   const S8Job &j = in_a ? a : b;
-  const uint64_t u = in_a ? t : t - items_a;
-  const uint32_t cpr = in_a ? cpr_a : cpr_b;
-  uint64_t r, q;
-  if (u <= 0xFFFFFFFFull) {
-    r = (uint32_t)u / cpr;
-    q = (uint32_t)u - (uint32_t)r * cpr;
-  } else {
-    r = u / cpr;
-    q = u - r * cpr;
-  }
-  const int64_t c = (int64_t)q * 4;
-  const int8_t *src = j.src + (int64_t)r * j.ld_src + c;
-  uint16_t *dst = j.dst + (int64_t)r * j.ld_dst + c;
-  if (c + 4 <= j.cols) {
-    uint32_t w;
-    if ((reinterpret_cast<uintptr_t>(src) & 3) == 0) {
-      w = __ldcs(reinterpret_cast<const unsigned int *>(src));
+  int64_t r, c;
+  piece_rc(in_a ? t : t - items_a, in_a ? cpr_a : cpr_b, 16, r, c);
+  const int8_t *src = j.src + r * j.ld_src + c;
+  uint16_t *dst = j.dst + r * j.ld_dst + c;
+  if (c + 16 <= j.cols) {
+    const uintptr_t al = reinterpret_cast<uintptr_t>(src);
+    int4 raw;
+    if ((al & 15) == 0) {
+      raw = __ldcs(reinterpret_cast<const int4 *>(src));
+    } else if ((al & 7) == 0) {
+      const int2 x = __ldcs(reinterpret_cast<const int2 *>(src)), y = __ldcs(reinterpret_cast<const int2 *>(src) + 1);
+      raw = make_int4(x.x, x.y, y.x, y.y);
+    } else if ((al & 3) == 0) {
+      const int *q = reinterpret_cast<const int *>(src);
+      raw = make_int4(__ldcs(q), __ldcs(q + 1), __ldcs(q + 2), __ldcs(q + 3));
     } else {
-      w = (uint32_t)(uint8_t)src[0] | ((uint32_t)(uint8_t)src[1] << 8) | ((uint32_t)(uint8_t)src[2] << 16) |
-          ((uint32_t)(uint8_t)src[3] << 24);
+      uint32_t w[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        w[i] = (uint32_t)(uint8_t)src[4 * i] | ((uint32_t)(uint8_t)src[4 * i + 1] << 8) |
+               ((uint32_t)(uint8_t)src[4 * i + 2] << 16) | ((uint32_t)(uint8_t)src[4 * i + 3] << 24);
+      raw = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
     }
-    uint32_t lo, hi;
-    s8x4_to_bf16x4(w, lo, hi);
-    *reinterpret_cast<uint2 *>(dst) = make_uint2(lo, hi);
+    uint4 lo, hi;
+    s8x16_to_bf16x16(raw, lo, hi);
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+    d[0] = lo;
+    d[1] = hi;
   } else {
     for (int64_t i = 0; c + i < j.cols; ++i) dst[i] = (uint16_t)s8_to_bf16_bits(src[i]);
   }
@@ -327,7 +345,7 @@ cudaError_t launch_s8_to_bf16_pair(const S8Job &a, const S8Job &b, int sms, cuda
     s8_to_bf16_dense_kernel<<<(unsigned)((vecs + kS8Threads - 1) / kS8Threads), kS8Threads, 0, st>>>(a, b, na, nb);
     return cudaGetLastError();
   }
-  const uint64_t cpr_a = (uint64_t)(a.cols + 3) / 4, cpr_b = (uint64_t)(b.cols + 3) / 4;
+  const uint64_t cpr_a = (uint64_t)(a.cols + 15) / 16, cpr_b = (uint64_t)(b.cols + 15) / 16;
   const uint64_t items_a = (uint64_t)a.rows * cpr_a, items = items_a + (uint64_t)b.rows * cpr_b;
   if (items == 0) return cudaSuccess;
   s8_to_bf16_pair_kernel<<<(unsigned)((items + kS8Threads - 1) / kS8Threads), kS8Threads, 0, st>>>(

@@ -189,6 +189,15 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
+// GEMM_ERR_CUDA, reporting the failing step (and CUDA's message) on stderr
+// when GB300_GEMM_DEBUG=1.
+gemm_status_t cuda_failed(const char *what, cudaError_t e = cudaSuccess) {
+  if (overrides().debug)
+    std::fprintf(stderr, "[gb300_gemm] %s failed%s%s\n", what, e != cudaSuccess ? ": " : "",
+                 e != cudaSuccess ? cudaGetErrorString(e) : "");
+  return GEMM_ERR_CUDA;
+}
+
 // 2-D bf16 tensor map: inner extent `inner` (contiguous), outer extent
 // `outer`, row pitch `ld` elements, box box_inner x box_outer, 128-byte
 // swizzle.  Out-of-range box elements read as zero.
@@ -394,14 +403,14 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
                      int64_t ldb, void *C, int64_t ldc, int esize, void *partials, cudaStream_t st) {
   TcParams &p = pl.p;
   CUtensorMap ta, tb;
-  if (!encode_bf16_2d(&ta, A, (uint64_t)p.K, (uint64_t)p.M, (uint64_t)lda, kBK, kBM)) return GEMM_ERR_CUDA;
+  if (!encode_bf16_2d(&ta, A, (uint64_t)p.K, (uint64_t)p.M, (uint64_t)lda, kBK, kBM)) return cuda_failed("A tensor map");
   // K-major B boxes cover the CTA's share of the tile width: all of it, or
   // half of it for a CTA pair.
   const uint32_t b_rows = pl.v.pair ? pl.v.bn / 2 : pl.v.bn;
   const bool ok_b = pl.v.b_kmajor
                         ? encode_bf16_2d(&tb, B, (uint64_t)p.K, (uint64_t)p.N, (uint64_t)ldb, kBK, b_rows)
                         : encode_bf16_2d(&tb, B, (uint64_t)p.N, (uint64_t)p.K, (uint64_t)ldb, 64, kBK);
-  if (!ok_b) return GEMM_ERR_CUDA;
+  if (!ok_b) return cuda_failed("B tensor map");
   p.C = C;
   p.ldc = ldc;
   p.c_vec = aligned16(C) && ((ldc * esize) % 16 == 0);
@@ -423,7 +432,7 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
       if (p.N % 4 == 0) {
         if (!encode_out(&tout, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, partials,
                         (uint64_t)p.N, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.splits))
-          return GEMM_ERR_CUDA;
+          return cuda_failed("partials tensor map");
         p.out_tma = kOutTmaWs;
       }
     } else if (p.c_vec) {
@@ -433,7 +442,7 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
                                                           : CU_TENSOR_MAP_DATA_TYPE_UINT8;
       if (!encode_out(&tout, type, (uint32_t)esize, C, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ldc, 1,
                       pl.v.tma_out == 2 ? 16 : 32))
-        return GEMM_ERR_CUDA;
+        return cuda_failed("C tensor map");
       p.out_tma = kOutTmaC;
     }
   }
@@ -449,7 +458,7 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
     e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, tout, p, pl.grid, st)
                             : launch_tc_bf16(pl.v, ta, tb, tout, p, pl.grid, st);
   g_launches.fetch_add(1);
-  if (e != cudaSuccess) return GEMM_ERR_CUDA;
+  if (e != cudaSuccess) return cuda_failed(pl.v.pair ? "CTA-pair kernel launch" : "tensor-core kernel launch", e);
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
   if (p.splits > 1) {
     e = pl.v.epi == kEpiS32
