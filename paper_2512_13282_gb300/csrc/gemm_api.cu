@@ -415,13 +415,18 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   p.ldc = ldc;
   p.c_vec = aligned16(C) && ((ldc * esize) % 16 == 0);
   p.ws = partials;
-  // Epilogue stores through TMA where the output allows it: bf16 or int32
-  // C with a 16-byte aligned base and pitch; split-K partials when their
-  // pitch (N words) is a multiple of 16 bytes.  int16 / int8 outputs and
-  // other cases store directly (GB300_GEMM_TMA_STORE=0 forces that).
+  // Epilogue stores through TMA where the output allows it: C with a
+  // 16-byte aligned base and pitch whose rows also END on a 16-byte
+  // boundary (N * esize a multiple of 16) -- a TMA store clipped at column N
+  // still writes the rest of the last 16-byte piece of each row, which for
+  // ldc > N lies in the caller's padding (measured on GB300: N = 5 bf16
+  // with ldc = 8 had columns 5..7 overwritten); split-K partials when their
+  // pitch (N words) is a multiple of 16 bytes.  Other cases store directly
+  // (GB300_GEMM_TMA_STORE=0 forces that).
   const bool s32 = pl.v.epi == kEpiS32;
   const bool tma_ok = overrides().tma_store &&
-                      (p.splits > 1 ? p.N % 4 == 0 && pl.v.tma_out == 1 : p.c_vec != 0);
+                      (p.splits > 1 ? p.N % 4 == 0 && pl.v.tma_out == 1
+                                    : p.c_vec != 0 && ((int64_t)p.N * esize) % 16 == 0);
   // An output that will be stored directly wants the variant with the extra
   // pipeline stage where one exists (int8 at 192 / 224).
   if (!tma_ok && s32 && (pl.v.bn == 192 || pl.v.bn == 224)) pl.v.tma_out = 0;

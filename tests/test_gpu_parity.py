@@ -119,6 +119,35 @@ def test_parity_leading_dims_and_offsets(dtype, layout, pads):
     _check(dtype, A, B, layout, C)
 
 
+@pytest.mark.parametrize("dtype", ["int8", "bf16", "int8_int16", "int8_int8"])
+@pytest.mark.parametrize("pair", ["0", "1"], ids=["single", "pair"])
+@pytest.mark.parametrize("N", [333, 5])
+def test_row_ends_inside_padded_pitch(dtype, pair, N, monkeypatch):
+    """C rows whose pitch is a multiple of 16 bytes but whose last element
+    is not at a 16-byte boundary (ldc > N): nothing of the padding between
+    column N and the pitch may be written (a TMA store clipped at N still
+    writes the rest of the row's last 16-byte piece, so such C is stored
+    directly).  The guard check of U.run covers the padding."""
+    monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", "0")
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    monkeypatch.setenv("GB300_GEMM_PAIR", pair)
+    M, K = 300, 777
+    esize = {"int8": 4, "bf16": 2, "int8_int16": 2, "int8_int8": 1}[dtype]
+    ldc = N + 1
+    while (ldc * esize) % 16:
+        ldc += 1
+    assert (N * esize) % 16 != 0
+    base = "bf16" if dtype == "bf16" else "int8"
+    A, B = _inputs(base, M, N, K, COL, seed=N + len(dtype))
+    shift = 9 if dtype in ("int8_int16", "int8_int8") else 0
+    C = U.run(dtype, A, B, COL, ldc=ldc, shift=shift)
+    if dtype in ("int8", "bf16"):
+        _check(dtype, A, B, COL, C)
+    else:
+        want = oracle.requantize(oracle.gemm_s8(A, B, COL), shift, 16 if dtype == "int8_int16" else 8)
+        assert np.array_equal(C.astype(np.int64), want)
+
+
 @pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
 def test_bf16_integer_inputs_bit_exact(layout):
     """Integer-valued inputs in [-8, 8]: fp32 accumulation is exact in any
