@@ -94,3 +94,82 @@ def test_fuzz(i, monkeypatch):
             want = oracle.requantize(want, shift, 16 if dtype == "int8_int16" else 8)
         bad = np.argwhere(C.astype(np.int64) != want)
         assert bad.size == 0, f"{len(bad)} mismatches, first at {bad[:5].tolist()}"
+
+
+def _case_small_operand(i):
+    """Shapes of the small-operand int8 kernel: one side of at most 128 rows
+    against a long other side, K across several 1024-deep slabs, B in both
+    layouts, with padded pitches (multiples of 16 bytes, so that the
+    operands stay TMA-legal) or odd ones (the general path then)."""
+    rng = np.random.default_rng(5000 + i)
+    small = int(rng.integers(1, 129))
+    big = int(rng.integers(129, 3000))
+    K = int(rng.integers(16, 6000))
+    if i % 3 == 2:  # N is the small side
+        M, N = big, small
+    else:
+        M, N = small, big
+    while M * N * K > 2e8:
+        K //= 2
+    layout = (ROW, COL)[i % 2]
+    out = ("int8", "int8_int16", "int8_int8")[(i // 2) % 3]
+    aligned = rng.uniform() < 0.7
+    pad = lambda n: (-n) % 16 + 16 * int(rng.integers(0, 2)) if aligned else int(rng.integers(0, 5))
+    return out, layout, M, N, K, pad, int(rng.integers(0, 12))
+
+
+SMALL_OPERAND = [_case_small_operand(i) for i in range(90)]
+
+
+@pytest.mark.parametrize("i", range(len(SMALL_OPERAND)),
+                         ids=[f"{c[0]}-{'Brow' if c[1] == ROW else 'Bcol'}-{c[2]}x{c[3]}x{c[4]}" for c in SMALL_OPERAND])
+def test_fuzz_small_operand(i, monkeypatch):
+    out, layout, M, N, K, pad, shift = SMALL_OPERAND[i]
+    for k in ROUTE_ENV:
+        monkeypatch.delenv(k, raising=False)
+    monkeypatch.setenv("GB300_GEMM_SKINNY_MAX_M", "0")
+    monkeypatch.setenv("GB300_GEMM_TINY_MAX_MACS", "0")
+    A = W.random_int8((M, K), 3 * i + 1)
+    B = W.random_int8((K, N) if layout == ROW else (N, K), 3 * i + 2)
+    bcols = N if layout == ROW else K
+    lda, ldb = K + pad(K), bcols + pad(bcols)
+    shift = shift if out != "int8" else 0
+    C = U.run(out, A, B, layout, lda=lda, ldb=ldb, shift=shift)
+    want = oracle.gemm_s8(A, B, layout)
+    if out != "int8":
+        want = oracle.requantize(want, shift, 16 if out == "int8_int16" else 8)
+    bad = np.argwhere(C.astype(np.int64) != want)
+    assert bad.size == 0, f"{len(bad)} mismatches, first at {bad[:5].tolist()}"
+
+
+def _case_noalloc(i):
+    rng = np.random.default_rng(9000 + i)
+    M, N, K = (int(np.exp(rng.uniform(np.log(lo), np.log(hi)))) for lo, hi in ((1, 700), (1, 900), (1, 3000)))
+    return M, N, K, (ROW, COL)[i % 2], int(rng.integers(0, 3))
+
+
+NOALLOC = [_case_noalloc(i) for i in range(24)]
+
+
+@pytest.mark.parametrize("i", range(len(NOALLOC)),
+                         ids=[f"{'Brow' if c[3] == ROW else 'Bcol'}-{c[0]}x{c[1]}x{c[2]}" for c in NOALLOC])
+def test_fuzz_noalloc(i):
+    """The no-allocation entry point on random shapes, padded pitches and
+    offsets, against the oracle."""
+    M, N, K, layout, pad = NOALLOC[i]
+    A = W.random_int8((M, K), 11 * i + 1)
+    B = W.random_int8((K, N) if layout == ROW else (N, K), 11 * i + 2)
+    bcols = N if layout == ROW else K
+    abuf, pa, lda = U.to_device(A, K + pad, pad)
+    bbuf, pb, ldb = U.to_device(B, bcols + pad, 0)
+    ldc = N + pad
+    C = torch.full((M * ldc + 16,), U.SENTINEL32, dtype=torch.int32, device="cuda")
+    st = G.gemm_s8s8_s32_noalloc(M, N, K, pa, lda, pb, ldb, layout, C.data_ptr(), ldc, 0)
+    assert st == G.GEMM_OK, G.gemm_status_string(st)
+    torch.cuda.synchronize()
+    assert G.gemm_device_status() == G.GEMM_OK
+    host = C.cpu().numpy()
+    body = host[:M * ldc].reshape(M, ldc)
+    assert (body[:, N:] == U.SENTINEL32).all() and (host[M * ldc:] == U.SENTINEL32).all()
+    assert np.array_equal(body[:, :N].astype(np.int64), oracle.gemm_s8(A, B, layout))
+    del abuf, bbuf
