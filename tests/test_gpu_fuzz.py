@@ -173,3 +173,76 @@ def test_fuzz_noalloc(i):
     assert (body[:, N:] == U.SENTINEL32).all() and (host[M * ldc:] == U.SENTINEL32).all()
     assert np.array_equal(body[:, :N].astype(np.int64), oracle.gemm_s8(A, B, layout))
     del abuf, bbuf
+
+
+def _case_large(i):
+    """More tiles than SMs (persistent loops over several rounds, group
+    rasterisation edges), with a forced family / width / split now and then."""
+    rng = np.random.default_rng(7000 + i)
+    M, N, K = int(rng.integers(1200, 3000)), int(rng.integers(1200, 3000)), int(rng.integers(200, 900))
+    dtype = ("int8", "bf16")[i % 2]
+    layout = (ROW, COL)[(i // 2) % 2]
+    env = {}
+    if i % 3 == 1:
+        env = {"GB300_GEMM_BN": str(int(rng.choice([128, 192, 224, 256]))),
+               "GB300_GEMM_PAIR": str(int(rng.integers(0, 2))), "GB300_GEMM_SPLITS": str(int(rng.integers(1, 4)))}
+    return dtype, layout, M, N, K, env
+
+
+LARGE = [_case_large(i) for i in range(12)]
+
+
+@pytest.mark.parametrize("i", range(len(LARGE)),
+                         ids=[f"{c[0]}-{'Brow' if c[1] == ROW else 'Bcol'}-{c[2]}x{c[3]}x{c[4]}" for c in LARGE])
+def test_fuzz_large(i, monkeypatch):
+    dtype, layout, M, N, K, env = LARGE[i]
+    for k in ROUTE_ENV:
+        monkeypatch.delenv(k, raising=False)
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
+    bshape = (K, N) if layout == ROW else (N, K)
+    if dtype == "bf16":
+        A, B = W.random_bf16((M, K), 13 * i + 1), W.random_bf16(bshape, 13 * i + 2)
+    else:
+        A, B = W.random_int8((M, K), 13 * i + 1), W.random_int8(bshape, 13 * i + 2)
+    C = U.run(dtype, A, B, layout)
+    if dtype == "bf16":
+        ref, mag = oracle.gemm_bf16(A, B, layout)
+        assert oracle.bf16_within_bound(C, ref, mag).all()
+        _check_rounding(C, ref)
+    else:
+        assert np.array_equal(C.astype(np.int64), oracle.gemm_s8(A, B, layout))
+
+
+def _case_aspect(i):
+    """Extreme aspect ratios: one of M, N, K tiny (1..16) against the others."""
+    rng = np.random.default_rng(8000 + i)
+    dims = [int(rng.integers(1, 17)), int(rng.integers(200, 4000)), int(rng.integers(200, 4000))]
+    rng.shuffle(dims)
+    M, N, K = dims
+    while M * N * K > 1.2e8:
+        K = max(1, K // 2)
+    return ("int8", "bf16")[i % 2], (ROW, COL)[(i // 2) % 2], M, N, K
+
+
+ASPECT = [_case_aspect(i) for i in range(40)]
+
+
+@pytest.mark.parametrize("i", range(len(ASPECT)),
+                         ids=[f"{c[0]}-{'Brow' if c[1] == ROW else 'Bcol'}-{c[2]}x{c[3]}x{c[4]}" for c in ASPECT])
+def test_fuzz_aspect(i, monkeypatch):
+    dtype, layout, M, N, K = ASPECT[i]
+    for k in ROUTE_ENV:
+        monkeypatch.delenv(k, raising=False)
+    bshape = (K, N) if layout == ROW else (N, K)
+    if dtype == "bf16":
+        A, B = W.random_bf16((M, K), 17 * i + 1), W.random_bf16(bshape, 17 * i + 2)
+    else:
+        A, B = W.random_int8((M, K), 17 * i + 1), W.random_int8(bshape, 17 * i + 2)
+    C = U.run(dtype, A, B, layout)
+    if dtype == "bf16":
+        ref, mag = oracle.gemm_bf16(A, B, layout)
+        assert oracle.bf16_within_bound(C, ref, mag).all()
+        _check_rounding(C, ref)
+    else:
+        assert np.array_equal(C.astype(np.int64), oracle.gemm_s8(A, B, layout))
