@@ -24,10 +24,14 @@
  *     validates, enqueues its kernels and returns without synchronising.
  *   - M == 0 or N == 0 is a no-op returning GEMM_OK; K == 0 writes zeros.
  *   - Errors are returned as status codes; nothing is thrown across the ABI.
- *   - The library keeps a lazily grown device workspace (for operand staging
- *     and split-K partials), allocated stream-ordered on first need and
- *     released by gemm_release_resources().  Calls on different streams that
- *     both need the workspace must be ordered by the caller.
+ *   - The library keeps lazily grown device scratch (operand staging copies,
+ *     split-K partials, the small-M kernel's counters), allocated
+ *     stream-ordered on first need, one set per stream: the first 16 streams
+ *     that call the library on a device keep theirs between calls, a call on
+ *     any further stream allocates its own and frees it (stream-ordered) when
+ *     it ends.  Calls on different streams may therefore run concurrently;
+ *     calls on one stream must not be issued from several host threads at
+ *     once.  gemm_release_resources() frees the scratch.
  *   - Environment variables that override the planner, for tests and
  *     benchmarks (int8 results are identical either way; bf16 results may
  *     differ in summation order, within the same accuracy): GB300_GEMM_BN,

@@ -28,14 +28,28 @@ namespace {
 constexpr int kMaxDevices = 64;
 constexpr int64_t kMaxExactK = 131071;  // 131072 * 2^14 = 2^31 overflows int32
 
-struct DeviceState {
-  bool ready = false;
-  int sms = 0;
-  uint32_t *err = nullptr;
+// Scratch of a call: operand staging copies, split-K partials, and the
+// small-M kernel's zeroed ticket counters.  Each stream that calls the
+// library on a device gets a scratch slot of its own (the first
+// kStreamSlots streams), kept between calls and grown stream-ordered on that
+// stream, so that calls on different streams never share device memory; a
+// call on a further stream allocates its scratch stream-ordered and frees it
+// at its end.
+constexpr int kStreamSlots = 16;
+struct Scratch {
+  bool owned = false;
+  cudaStream_t owner = nullptr;
   void *ws = nullptr;
   size_t ws_bytes = 0;
   uint32_t *tickets = nullptr;  // zeroed counters of the small-M kernel
   size_t tickets_count = 0;
+};
+
+struct DeviceState {
+  bool ready = false;
+  int sms = 0;
+  uint32_t *err = nullptr;
+  Scratch slots[kStreamSlots];
 };
 
 std::mutex g_mu;
@@ -148,42 +162,88 @@ gemm_status_t device_state(DeviceState **out) {
   return GEMM_OK;
 }
 
-// Grow the device workspace (stream-ordered) to at least `bytes`.
-gemm_status_t ensure_workspace(DeviceState &d, size_t bytes, cudaStream_t st) {
-  if (bytes <= d.ws_bytes) return GEMM_OK;
-  std::lock_guard<std::mutex> lk(g_mu);
-  if (bytes <= d.ws_bytes) return GEMM_OK;
-  if (d.ws) {
-    if (cudaFreeAsync(d.ws, st) != cudaSuccess) return GEMM_ERR_CUDA;
-    d.ws = nullptr;
-    d.ws_bytes = 0;
+// The scratch of the call in progress on this host thread (set by ScratchLease).
+thread_local Scratch *t_scratch = nullptr;
+
+// Holds the calling stream's scratch for the duration of one call: its own
+// slot, or (more streams than slots) a scratch of this call alone, freed
+// stream-ordered when the call ends.
+class ScratchLease {
+ public:
+  ScratchLease(DeviceState &d, cudaStream_t st) : st_(st) {
+    {
+      std::lock_guard<std::mutex> lk(g_mu);
+      for (Scratch &x : d.slots)
+        if (x.owned && x.owner == st) {
+          s_ = &x;
+          break;
+        }
+      if (!s_)
+        for (Scratch &x : d.slots)
+          if (!x.owned) {
+            x.owned = true;
+            x.owner = st;
+            s_ = &x;
+            break;
+          }
+    }
+    if (!s_) s_ = &temp_;
+    t_scratch = s_;
+  }
+  ~ScratchLease() {
+    if (s_ == &temp_) {
+      if (temp_.ws) cudaFreeAsync(temp_.ws, st_);
+      if (temp_.tickets) cudaFreeAsync(temp_.tickets, st_);
+    }
+    t_scratch = nullptr;
+  }
+  ScratchLease(const ScratchLease &) = delete;
+  ScratchLease &operator=(const ScratchLease &) = delete;
+
+ private:
+  cudaStream_t st_;
+  Scratch *s_ = nullptr;
+  Scratch temp_;
+};
+
+// Grow the current call's workspace (stream-ordered, on its own stream) to
+// at least `bytes`; the result is scratch_ws().
+gemm_status_t ensure_workspace(size_t bytes, cudaStream_t st) {
+  Scratch &s = *t_scratch;
+  if (bytes <= s.ws_bytes) return GEMM_OK;
+  if (s.ws) {
+    if (cudaFreeAsync(s.ws, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    s.ws = nullptr;
+    s.ws_bytes = 0;
   }
   const size_t grown = bytes + bytes / 4;
-  if (cudaMallocAsync(&d.ws, grown, st) != cudaSuccess) {
-    d.ws = nullptr;
+  if (cudaMallocAsync(&s.ws, grown, st) != cudaSuccess) {
+    s.ws = nullptr;
     return GEMM_ERR_CUDA;
   }
-  d.ws_bytes = grown;
+  s.ws_bytes = grown;
   return GEMM_OK;
 }
+void *scratch_ws() { return t_scratch->ws; }
 
-// Grow the zeroed ticket counters of the small-M kernel to `count`.
-gemm_status_t ensure_tickets(DeviceState &d, size_t count, cudaStream_t st) {
-  if (count <= d.tickets_count) return GEMM_OK;
-  std::lock_guard<std::mutex> lk(g_mu);
-  if (count <= d.tickets_count) return GEMM_OK;
-  if (d.tickets && cudaFreeAsync(d.tickets, st) != cudaSuccess) return GEMM_ERR_CUDA;
-  d.tickets = nullptr;
-  d.tickets_count = 0;
+// Grow the current call's zeroed ticket counters of the small-M kernel to
+// `count` (the kernel leaves them zero again).
+gemm_status_t ensure_tickets(size_t count, cudaStream_t st) {
+  Scratch &s = *t_scratch;
+  if (count <= s.tickets_count) return GEMM_OK;
+  if (s.tickets && cudaFreeAsync(s.tickets, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  s.tickets = nullptr;
+  s.tickets_count = 0;
   const size_t n = count < 1024 ? 1024 : count;
-  if (cudaMallocAsync(reinterpret_cast<void **>(&d.tickets), n * sizeof(uint32_t), st) != cudaSuccess ||
-      cudaMemsetAsync(d.tickets, 0, n * sizeof(uint32_t), st) != cudaSuccess) {
-    d.tickets = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&s.tickets), n * sizeof(uint32_t), st) != cudaSuccess ||
+      cudaMemsetAsync(s.tickets, 0, n * sizeof(uint32_t), st) != cudaSuccess) {
+    s.tickets = nullptr;
     return GEMM_ERR_CUDA;
   }
-  d.tickets_count = n;
+  s.tickets_count = n;
   return GEMM_OK;
 }
+uint32_t *scratch_tickets() { return t_scratch->tickets; }
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -523,10 +583,10 @@ gemm_status_t run_skinny(DeviceState &d, int64_t M, int64_t N, int64_t K, const 
   p.b_align = (int)(bits & (~bits + 1));  // lowest set bit: 1, 2, 4, 8 or 16
   gemm_status_t s;
   if (p.ks > 1) {
-    if ((s = ensure_workspace(d, (size_t)p.ks * M * N * 4, st)) != GEMM_OK) return s;
-    if ((s = ensure_tickets(d, (size_t)strips, st)) != GEMM_OK) return s;
-    p.ws = d.ws;
-    p.tickets = d.tickets;
+    if ((s = ensure_workspace((size_t)p.ks * M * N * 4, st)) != GEMM_OK) return s;
+    if ((s = ensure_tickets((size_t)strips, st)) != GEMM_OK) return s;
+    p.ws = scratch_ws();
+    p.tickets = scratch_tickets();
   }
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
@@ -548,6 +608,7 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   DeviceState *d = nullptr;
   if ((s = device_state(&d)) != GEMM_OK) return s;
+  const ScratchLease lease(*d, st);
   if (K == 0) {
     g_launches.fetch_add(1);
     return launch_zero_fill(C, M, N, ldc, 2, d->sms, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
@@ -568,8 +629,8 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
   if (pack_b) { L.b_off = off; off = align_up(off + (size_t)b_rows * ldb_p * 2, 256); }
   if (pl.p.splits > 1) { L.part_off = off; off = align_up(off + (size_t)pl.p.splits * M * N * 4, 256); }
   L.total = off;
-  if (L.total && (s = ensure_workspace(*d, L.total, st)) != GEMM_OK) return s;
-  uint8_t *ws = static_cast<uint8_t *>(d->ws);
+  if (L.total && (s = ensure_workspace(L.total, st)) != GEMM_OK) return s;
+  uint8_t *ws = static_cast<uint8_t *>(scratch_ws());
   const uint16_t *Au = A, *Bu = B;
   int64_t lda_u = lda, ldb_u = ldb;
   if (pack_a) {
@@ -669,11 +730,11 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   const bool add_into_c = splits > 1 && out_bits == 32;
   const size_t q_bytes = align_up(s8tm_q_image_bytes(qn, Q_rows, K), 256);
   const size_t total = q_bytes + (splits > 1 && !add_into_c ? (size_t)splits * M * N * 4 : 0);
-  if ((s = ensure_workspace(d, total, st)) != GEMM_OK) {
+  if ((s = ensure_workspace(total, st)) != GEMM_OK) {
     *status = s;
     return true;
   }
-  uint8_t *ws = static_cast<uint8_t *>(d.ws);
+  uint8_t *ws = static_cast<uint8_t *>(scratch_ws());
   *status = GEMM_ERR_CUDA;
   g_launches.fetch_add(1);
   if (launch_s8tm_stage_q(Qs, sq, sk, Q_rows, K, qn, ws, add_into_c ? static_cast<int32_t *>(C) : nullptr, M, N,
@@ -741,6 +802,7 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   DeviceState *d = nullptr;
   if ((s = device_state(&d)) != GEMM_OK) return s;
+  const ScratchLease lease(*d, st);
   const int out_esize = out_bits / 8;
   if (K == 0) {  // every sum is 0, and 0 requantises to 0
     g_launches.fetch_add(1);
@@ -773,8 +835,8 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   off = align_up(off + (size_t)b_rows * ldb_p * 2, 256);
   if (pl.p.splits > 1) { L.part_off = off; off = align_up(off + (size_t)pl.p.splits * M * N * 4, 256); }
   L.total = off;
-  if ((s = ensure_workspace(*d, L.total, st)) != GEMM_OK) return s;
-  uint8_t *ws = static_cast<uint8_t *>(d->ws);
+  if ((s = ensure_workspace(L.total, st)) != GEMM_OK) return s;
+  uint8_t *ws = static_cast<uint8_t *>(scratch_ws());
   uint16_t *Ab = reinterpret_cast<uint16_t *>(ws + L.a_off);
   uint16_t *Bb = reinterpret_cast<uint16_t *>(ws + L.b_off);
   g_launches.fetch_add(1);
@@ -837,12 +899,11 @@ void gemm_release_resources(void) {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return;
   std::lock_guard<std::mutex> lk(g_mu);
   DeviceState &d = g_dev[dev];
-  if (d.ws) cudaFree(d.ws);
-  d.ws = nullptr;
-  d.ws_bytes = 0;
-  if (d.tickets) cudaFree(d.tickets);
-  d.tickets = nullptr;
-  d.tickets_count = 0;
+  for (Scratch &x : d.slots) {
+    if (x.ws) cudaFree(x.ws);
+    if (x.tickets) cudaFree(x.tickets);
+    x = Scratch{};
+  }
   d.ready = false;  // look the device's symbols up again at the next call
   noalloc_forget_device(dev);
 }
