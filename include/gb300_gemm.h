@@ -32,6 +32,12 @@
  *     it ends.  Calls on different streams may therefore run concurrently;
  *     calls on one stream must not be issued from several host threads at
  *     once.  gemm_release_resources() frees the scratch.
+ *   - CUDA graphs: calls may be captured on a stream that has already run,
+ *     outside capture, calls needing at least as much scratch (the same
+ *     shapes, say); a captured call that would need more returns
+ *     GEMM_ERR_UNSUPPORTED before enqueuing anything.  Scratch that a graph
+ *     refers to stays allocated until gemm_release_resources(), after which
+ *     graphs captured before must not be launched.
  *   - Environment variables that override the planner, for tests and
  *     benchmarks (int8 results are identical either way; bf16 results may
  *     differ in summation order, within the same accuracy): GB300_GEMM_BN,

@@ -11,6 +11,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include "gb300_gemm.h"
 #include "gemm_internal.h"
@@ -43,6 +44,11 @@ struct Scratch {
   size_t ws_bytes = 0;
   uint32_t *tickets = nullptr;  // zeroed counters of the small-M kernel
   size_t tickets_count = 0;
+  // Once a call has been captured into a CUDA graph, the graph refers to
+  // this scratch: buffers replaced by growth are then kept (not freed) until
+  // gemm_release_resources(), so that the graph stays valid.
+  bool captured = false;
+  std::vector<void *> retired;
 };
 
 struct DeviceState {
@@ -206,13 +212,43 @@ class ScratchLease {
   Scratch temp_;
 };
 
+// Whether `st` is being captured into a CUDA graph.
+bool capturing(cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  return cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs != cudaStreamCaptureStatusNone;
+}
+
+// Scratch of a stream's own slot needed by a call being captured into a
+// CUDA graph: it must exist already (the stream has run a call at least as
+// large before the capture), since memory allocated inside the capture
+// would belong to the graph alone.  (A stream without a slot of its own --
+// more streams than slots -- allocates inside the graph and frees there,
+// which the graph owns.)
+gemm_status_t scratch_for_capture(Scratch &s, bool enough) {
+  if (!enough) return GEMM_ERR_UNSUPPORTED;
+  s.captured = true;
+  return GEMM_OK;
+}
+
+// Release a buffer replaced by growth: stream-ordered, or kept while a
+// captured graph may still refer to it.
+gemm_status_t retire(Scratch &s, void *p, cudaStream_t st) {
+  if (!p) return GEMM_OK;
+  if (s.captured) {
+    s.retired.push_back(p);
+    return GEMM_OK;
+  }
+  return cudaFreeAsync(p, st) == cudaSuccess ? GEMM_OK : GEMM_ERR_CUDA;
+}
+
 // Grow the current call's workspace (stream-ordered, on its own stream) to
 // at least `bytes`; the result is scratch_ws().
 gemm_status_t ensure_workspace(size_t bytes, cudaStream_t st) {
   Scratch &s = *t_scratch;
+  if (capturing(st) && s.owned) return scratch_for_capture(s, bytes <= s.ws_bytes);
   if (bytes <= s.ws_bytes) return GEMM_OK;
   if (s.ws) {
-    if (cudaFreeAsync(s.ws, st) != cudaSuccess) return GEMM_ERR_CUDA;
+    if (retire(s, s.ws, st) != GEMM_OK) return GEMM_ERR_CUDA;
     s.ws = nullptr;
     s.ws_bytes = 0;
   }
@@ -230,8 +266,9 @@ void *scratch_ws() { return t_scratch->ws; }
 // `count` (the kernel leaves them zero again).
 gemm_status_t ensure_tickets(size_t count, cudaStream_t st) {
   Scratch &s = *t_scratch;
+  if (capturing(st) && s.owned) return scratch_for_capture(s, count <= s.tickets_count);
   if (count <= s.tickets_count) return GEMM_OK;
-  if (s.tickets && cudaFreeAsync(s.tickets, st) != cudaSuccess) return GEMM_ERR_CUDA;
+  if (retire(s, s.tickets, st) != GEMM_OK) return GEMM_ERR_CUDA;
   s.tickets = nullptr;
   s.tickets_count = 0;
   const size_t n = count < 1024 ? 1024 : count;
@@ -902,6 +939,7 @@ void gemm_release_resources(void) {
   for (Scratch &x : d.slots) {
     if (x.ws) cudaFree(x.ws);
     if (x.tickets) cudaFree(x.tickets);
+    for (void *p : x.retired) cudaFree(p);
     x = Scratch{};
   }
   d.ready = false;  // look the device's symbols up again at the next call
