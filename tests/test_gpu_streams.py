@@ -148,3 +148,62 @@ def test_streams_stress_against_single_calls():
     assert G.gemm_device_status() == G.GEMM_OK
     bad = [k for k, (a, b) in enumerate(zip(alone, together)) if not torch.equal(a, b)]
     assert not bad, f"{len(bad)} of {len(items)} concurrent GEMMs differ from the same GEMM run alone"
+
+
+def test_host_threads_each_with_a_stream():
+    """Four host threads, each issuing GEMMs on a stream of its own at the
+    same time (the binding releases the interpreter lock inside each call):
+    every result equals the same GEMM run alone."""
+    import threading
+    G.gemm_reload_overrides()
+    jobs = [("int8", 700, 800, 3000, COL), ("bf16", 200, 300, 6000, ROW), ("int8", 4, 3000, 3000, ROW),
+            ("int8", 96, 3000, 2048, COL)]
+    per_thread = []
+    for t in range(4):
+        items = []
+        for j, (dtype, M, N, K, layout) in enumerate(jobs):
+            seed = 50 * t + j
+            bsh = (K, N) if layout == ROW else (N, K)
+            if dtype == "int8":
+                tA = torch.from_numpy(W.random_int8((M, K), seed)).cuda()
+                tB = torch.from_numpy(W.random_int8(bsh, seed + 1)).cuda()
+                fn, cdt = G.gemm_s8s8_s32, torch.int32
+            else:
+                tA = torch.from_numpy(W.random_bf16((M, K), seed).view(np.int16)).cuda()
+                tB = torch.from_numpy(W.random_bf16(bsh, seed + 1).view(np.int16)).cuda()
+                fn, cdt = G.gemm_bf16_f32acc_bf16, torch.int16
+            items.append((fn, cdt, M, N, K, layout, tA, tB))
+        per_thread.append(items)
+
+    def call(it, stream):
+        fn, cdt, M, N, K, layout, tA, tB = it
+        C = torch.zeros((M, N), dtype=cdt, device="cuda")
+        st = fn(M, N, K, tA.data_ptr(), K, tB.data_ptr(), N if layout == ROW else K, layout, C.data_ptr(), N,
+                stream.cuda_stream)
+        return st, C
+
+    cur = torch.cuda.current_stream()
+    alone = [[call(it, cur)[1] for it in items] for items in per_thread]
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream() for _ in range(4)]
+    results = [None] * 4
+    start = threading.Barrier(4)
+
+    def worker(t):
+        start.wait()
+        out = []
+        for _ in range(3):
+            out += [call(it, streams[t]) for it in per_thread[t]]
+        results[t] = out
+
+    threads = [threading.Thread(target=worker, args=(t,)) for t in range(4)]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    torch.cuda.synchronize()
+    assert G.gemm_device_status() == G.GEMM_OK
+    for t in range(4):
+        for k, (st, C) in enumerate(results[t]):
+            assert st == G.GEMM_OK
+            assert torch.equal(C, alone[t][k % len(jobs)]), (t, k)
