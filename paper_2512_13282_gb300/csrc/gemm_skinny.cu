@@ -161,6 +161,11 @@ __global__ void __launch_bounds__(kSkThreads, BPS) skinny_rowB_kernel(const Skin
   constexpr int esize = INT8 ? 1 : 2;
   extern __shared__ uint32_t sk_smem[];
   __shared__ uint32_t ticket;
+  // launched with programmatic dependent launch: the next kernel of the
+  // stream may be scheduled now, and this one touches global memory only
+  // once the previous one has completed
+  griddep_launch_dependents();
+  griddep_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n0 = (int64_t)blockIdx.x * kCols;
   const int64_t k0 = (int64_t)blockIdx.y * p.kb;
@@ -335,6 +340,8 @@ __global__ void __launch_bounds__(kSkThreads, colb_blocks(MT)) skinny_colB_kerne
   constexpr int kElems = INT8 ? 16 : 8;            // elements per 16-byte chunk
   extern __shared__ uint32_t sk_smem[];
   __shared__ uint32_t ticket;
+  griddep_launch_dependents();  // programmatic dependent launch, as above
+  griddep_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n0 = (int64_t)blockIdx.x * kCols;
   const int64_t k0 = (int64_t)blockIdx.y * p.kb;
@@ -456,7 +463,8 @@ cudaError_t launch_mt(const SkinnyParams &p, dim3 grid, bool row_b, cudaStream_t
     auto kern = skinny_rowB_kernel<MT, VB, INT8, sh.rb, sh.bps>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kSkThreads, smem, st>>>(p);
+    e = launch_ex(kern, grid, dim3(kSkThreads), smem, st, 1, p);
+    if (e != cudaSuccess) return e;
   } else {
     const int kelems = INT8 ? 16 : 8;
     const size_t a_bytes = (size_t)MT * ((p.kb + kelems - 1) / kelems) * 16;
@@ -465,7 +473,8 @@ cudaError_t launch_mt(const SkinnyParams &p, dim3 grid, bool row_b, cudaStream_t
     auto kern = skinny_colB_kernel<MT, INT8>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kSkThreads, smem, st>>>(p);
+    e = launch_ex(kern, grid, dim3(kSkThreads), smem, st, 1, p);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

@@ -56,6 +56,11 @@ template <bool ROW_B>
 __global__ void __launch_bounds__(kTThreads) gemm_tiny_s8_kernel(const TinyParams p) {
   __shared__ uint32_t As[kTT][kTPad];
   __shared__ uint32_t Bs[kTT][kTPad];
+  // launched with programmatic dependent launch: the next kernel of the
+  // stream may be scheduled now; global memory is touched only once the
+  // previous kernel has completed
+  griddep_launch_dependents();
+  griddep_wait();
   const int tid = threadIdx.x;
   const int ty = tid >> 4, tx = tid & 15;
   const int64_t m0 = (int64_t)blockIdx.y * kTT, n0 = (int64_t)blockIdx.x * kTT;
@@ -158,11 +163,8 @@ __global__ void __launch_bounds__(kTThreads) gemm_tiny_s8_kernel(const TinyParam
 
 cudaError_t launch_tiny_s8(const TinyParams &p, bool row_b, cudaStream_t st) {
   const dim3 grid((unsigned)((p.N + kTT - 1) / kTT), (unsigned)((p.M + kTT - 1) / kTT));
-  if (row_b)
-    gemm_tiny_s8_kernel<true><<<grid, kTThreads, 0, st>>>(p);
-  else
-    gemm_tiny_s8_kernel<false><<<grid, kTThreads, 0, st>>>(p);
-  return cudaGetLastError();
+  return row_b ? launch_ex(gemm_tiny_s8_kernel<true>, grid, dim3(kTThreads), 0, st, 1, p)
+               : launch_ex(gemm_tiny_s8_kernel<false>, grid, dim3(kTThreads), 0, st, 1, p);
 }
 
 }  // namespace gb300
