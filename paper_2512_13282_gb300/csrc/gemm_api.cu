@@ -361,11 +361,14 @@ struct Plan {
 //   rounds * (kb_per_unit * kstep + unit) + split terms
 // (Eq. 9 with wave quantisation), with the per-variant K-step and unit costs
 // and the split constants fitted to measurements on GB300 (plan_table.h,
-// generated by tile_model.py).  The least time wins; on a tie the earlier
-// candidate (single CTA before pair, wider before narrower, fewer splits
-// before more).  tile_model.choose_plan is the same rule.  The DRAM time of
-// Eq. 6-8 and 10 (dram_us) classifies the GEMM but does not rank plans: with
-// the 129 MB L2 supplying the reuse, it barely depends on the tile.
+// generated by tile_model.py).  Plans are ranked by that time plus the share
+// kMemWeight of the DRAM time of Eq. 6-8 and 10 (dram_us) that the kernels
+// do not hide: with the 129 MB L2 supplying the reuse it separates plans
+// only where B is re-read once per group of row tiles (B does not stay in
+// L2 beside A and C), which CTA pairs do half as often.  The least rank
+// wins; on a tie the earlier candidate (single CTA before pair, wider before
+// narrower, fewer splits before more).  tile_model.choose_plan is the same
+// rule.
 double modelled_us(int64_t M, int64_t N, bool int8, bool pair, int bn, int64_t splits, int64_t kb_per,
                    int64_t rounds) {
   const int wi = bn == 128 ? 0 : bn == 192 ? 1 : bn == 224 ? 2 : 3;
@@ -377,17 +380,18 @@ double modelled_us(int64_t M, int64_t N, bool int8, bool pair, int bn, int64_t s
 }
 
 // Eq. 6-8 and 10: DRAM bytes of A (once: the grouped raster keeps a group's
-// 8 row tiles of A in L2 while it sweeps N), B (once if it, or A and B
-// together, fit in L2, else once per group of 8 row tiles) and C, at the
-// copy bandwidth, in microseconds.
+// 8 row tiles of A in L2 while it sweeps N), B (once if it fits in half the
+// L2 or A, B and C together fit in L2 -- C passes through L2 as the tiles
+// store it -- else once per group of 8 row tiles) and C, at the copy
+// bandwidth, in microseconds.
 double dram_us(int64_t M, int64_t N, int64_t K, bool int8, bool pair) {
-  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * K * N;
+  const double a_bytes = 2.0 * M * K, b_bytes = 2.0 * K * N, c_bytes = (double)M * N * (int8 ? 4 : 2);
   double rb = 1.0;
-  if (!(b_bytes <= plan_table::kL2Bytes / 2 || a_bytes + b_bytes <= plan_table::kL2Bytes)) {
+  if (!(b_bytes <= plan_table::kL2Bytes / 2 || a_bytes + b_bytes + c_bytes <= plan_table::kL2Bytes)) {
     rb = (double)ceil_div(M, 8 * (pair ? 2 * kBM : kBM));
     if (rb < 1.0) rb = 1.0;
   }
-  return (a_bytes + b_bytes * rb + (double)M * N * (int8 ? 4 : 2)) / (plan_table::kHbmGBs * 1e3);
+  return (a_bytes + b_bytes * rb + c_bytes) / (plan_table::kHbmGBs * 1e3);
 }
 
 Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms, int pairs) {
@@ -401,7 +405,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
   bool best_pair = false;
   int best_bn = 128;
   int64_t best_splits = 1;
-  double best_cost = -1.0;
+  double best_cost = -1.0, best_model = 0.0;
   for (int fam = 0; fam < 2; ++fam) {
     const bool pair = fam == 1;
     if (pair && (M <= kBM || pairs <= 0)) continue;  // the second CTA would only compute padding
@@ -432,9 +436,11 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
           if (s2 > 1 && (kb_per < 4 || tiles * s2 > 2 * slots)) continue;
         }
         seen[nseen++] = s2;
-        const double cost = modelled_us(M, N, int8, pair, bn, s2, kb_per, ceil_div(tiles * s2, slots));
+        const double model = modelled_us(M, N, int8, pair, bn, s2, kb_per, ceil_div(tiles * s2, slots));
+        const double cost = model + plan_table::kMemWeight * dram_us(M, N, K, int8, pair);
         if (best_cost < 0 || cost < best_cost - 1e-9) {
           best_cost = cost;
+          best_model = model;
           best_pair = pair;
           best_bn = bn;
           best_splits = s2;
@@ -462,7 +468,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
   else
     tma_out = ((bn != 224 && bn != 192) || kb_per <= 128) ? 1 : 0;
   pl.v = TcVariant{bn, b_kmajor, epi, pair, tma_out};
-  pl.model_us = best_cost;
+  pl.model_us = best_model;
   TcParams &p = pl.p;
   p.M = (int)M;
   p.N = (int)N;
@@ -486,7 +492,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
                  (long long)M, (long long)N, (long long)K, epi == kEpiS32 ? "int8" : "bf16",
                  b_kmajor ? "col" : "row", pair ? "pair" : "single", bn,
                  tma_out == 2 ? " tma-store-1k" : tma_out ? " tma-store" : "", (long long)tiles_m,
-                 (long long)tiles_n, (long long)splits, pl.grid, best_cost, sms, pairs);
+                 (long long)tiles_n, (long long)splits, pl.grid, best_model, sms, pairs);
   return pl;
 }
 

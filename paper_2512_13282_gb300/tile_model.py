@@ -43,12 +43,15 @@ pipeline stage, accumulating in TMEM.  The restatement:
   reduction launch: T_split = r0 + r1 * (4 * S * M * N bytes).
 
 With the 129 MB L2 supplying the reuse, T_mem hardly depends on the tile
-(unlike the NPU's, where m_ct and n_ct set the DRAM traffic directly), so it
-classifies a GEMM (compute- or memory-bound, the paper's balance) but does
-not rank plans.  The planner (csrc/gemm_api.cu make_plan) minimises
-T_comp + T_split over (family, BN, S) with the per-variant t_kstep and t_unit and the
-split constants that fit() derives from measurements (tile_sweep.py) and
-header_text() writes to csrc/plan_table.h.  balanced_search() is the paper's
+(unlike the NPU's, where m_ct and n_ct set the DRAM traffic directly): it
+classifies a GEMM (compute- or memory-bound, the paper's balance), and
+separates plans only where B does not stay in L2 beside A and C and is
+re-read once per group of row tiles (half as often with CTA pairs).  The
+planner (csrc/gemm_api.cu make_plan) minimises T_comp + T_split + w * T_mem
+over (family, BN, S) with the per-variant t_kstep and t_unit, the split
+constants and the weight w of the DRAM time that the kernels do not hide,
+which fit() derives from measurements (tile_sweep.py) and header_text()
+writes to csrc/plan_table.h.  balanced_search() is the paper's
 iterative procedure on the same candidates: the model proposes, measurements
 decide, and the walk stops at the first slowdown.
 
@@ -216,17 +219,19 @@ def candidate_plans(M, N, K, b_kmajor, sms=None, pair_slots=None):
 def mem_time_us(M, N, K, dtype, plan):
     """Eq. 6-8 and 10 for one plan, in microseconds: A once (the grouped
     raster keeps a group's 8 row tiles of A in L2 while it sweeps N), B once
-    if it (or A and B together) fits in L2, else once per group of 8 row
-    tiles (128 or 256 rows each: CTA pairs halve the re-reads), C once.
-    Split-K partials are left out: they stay in L2, and their cost is the
-    fitted split term."""
+    if it fits in half the L2 or A, B and C together fit in L2 (C passes
+    through L2 as the tiles store it), else once per group of 8 row tiles
+    (128 or 256 rows each: CTA pairs halve the re-reads), C once.  Split-K
+    partials are left out: they stay in L2, and their cost is the fitted
+    split term."""
     ty = 2  # operands are bf16 in the kernel (int8 is staged as bf16)
     tyc = 4 if dtype == "int8" else 2
     l2 = GB300["l2_bytes"]
-    a_bytes, b_bytes = M * K * ty, K * N * ty
+    a_bytes, b_bytes, c_bytes = M * K * ty, K * N * ty, M * N * tyc
     rows_per_group = 8 * (2 * BM if plan["pair"] else BM)
-    rb = 1.0 if (b_bytes <= l2 / 2 or a_bytes + b_bytes <= l2) else max(1.0, float(_ceil(M, rows_per_group)))
-    return (a_bytes + b_bytes * rb + M * N * tyc) / (GB300["hbm_gbs"] * 1e3)
+    fits = b_bytes <= l2 / 2 or a_bytes + b_bytes + c_bytes <= l2
+    rb = 1.0 if fits else max(1.0, float(_ceil(M, rows_per_group)))
+    return (a_bytes + b_bytes * rb + c_bytes) / (GB300["hbm_gbs"] * 1e3)
 
 
 def plan_cost_us(M, N, K, dtype, plan, table):
@@ -249,12 +254,20 @@ def group_key(dtype, pair, bn):
     return f"{dtype}/{'pair' if pair else 'single'}/{bn}"
 
 
+def rank_us(M, N, K, dtype, plan, table):
+    """What the planner minimises: T_comp + T_split plus the share
+    `mem_weight` of Eq. 10's DRAM time that the kernels do not hide -- which
+    separates plans only where B is re-read (B does not stay in L2 beside A
+    and C, and a CTA pair's 256-row groups re-read it half as often)."""
+    return plan_cost_us(M, N, K, dtype, plan, table) + table.get("mem_weight", 0.0) * mem_time_us(M, N, K, dtype, plan)
+
+
 def choose_plan(M, N, K, dtype, b_kmajor, table, sms=None, pair_slots=None):
-    """The planner: the candidate of least modelled time (the first one, in
+    """The planner: the candidate of least rank_us (the first one, in
     candidate order, on a tie)."""
     best, best_c = None, math.inf
     for p in candidate_plans(M, N, K, b_kmajor, sms, pair_slots):
-        c = plan_cost_us(M, N, K, dtype, p, table)
+        c = rank_us(M, N, K, dtype, p, table)
         if c < best_c - 1e-9:
             best, best_c = p, c
     return best
@@ -312,12 +325,25 @@ def fit(meas):
     for d, name in ((0, "bf16"), (1, "int8")):
         table["split"][name] = {"fixed_us": float(max(x[base + 2 * ng + 2 * d], 0.0)),
                                 "us_per_mb": float(max(x[base + 2 * ng + 2 * d + 1], 0.0))}
+    # The weight of the DRAM time in the ranking: the grid value in the
+    # middle of the run of values whose choices take the least measured time
+    # over the sweep (the choices change only at a few thresholds).
+    totals = []
+    for w in MEM_WEIGHTS:
+        table["mem_weight"] = w
+        totals.append(sum(r["model_us"] if r["model_us"] is not None else math.inf for r in evaluate(meas, table)))
+    least = min(totals)
+    run = [i for i, t in enumerate(totals) if t <= least + 1e-6]
+    table["mem_weight"] = MEM_WEIGHTS[run[len(run) // 2]]
     pred = np.array(rows) @ x
     rel = (pred - np.array(rhs)) / np.array(rhs)
     table["fit"] = {"plans": len(rhs), "shapes": len(shapes), "rms_rel_err": float(np.sqrt(np.mean(rel ** 2))),
                     "median_abs_rel_err": float(np.median(np.abs(rel))),
                     "max_abs_rel_err": float(np.max(np.abs(rel)))}
     return table
+
+
+MEM_WEIGHTS = (0.0, 0.025, 0.05, 0.1, 0.2, 0.4)
 
 
 def predict_us(M, N, K, dtype, plan, table):
@@ -389,7 +415,8 @@ def header_text(table, source="plan_measurements.json"):
         "// epilogue), in microseconds; and per operand type the split-K terms",
         "// (reduction launch, and time per MB of fp32/int32 partials).  The planner",
         "// minimises rounds * (K steps per unit * kstep + unit) + split terms",
-        "// (Eq. 9 with wave quantisation), against the DRAM time of Eq. 6-8, 10.",
+        "// (Eq. 9 with wave quantisation) + kMemWeight * the DRAM time of Eq. 6-8,",
+        "// 10 (the share of B's re-reads the kernels do not hide).",
         "#pragma once",
         "",
         "namespace gb300 {",
@@ -424,6 +451,7 @@ def header_text(table, source="plan_measurements.json"):
         "// Eq. 10: DRAM bandwidth (GB/s) and the L2 capacity the reuse factors use.",
         "constexpr double kHbmGBs = %.1f;" % GB300["hbm_gbs"],
         "constexpr double kL2Bytes = %.1f;" % GB300["l2_bytes"],
+        "constexpr double kMemWeight = %.3f;" % table["mem_weight"],
         "",
         "}  // namespace plan_table",
         "}  // namespace gb300",
@@ -448,6 +476,7 @@ def table_from_header(text):
     fx = [float(x) for x in re.findall(r"kSplitFixedUs\[2\] = \{([0-9.]+)f, ([0-9.]+)f\}", text)[0]]
     pm = [float(x) for x in re.findall(r"kSplitUsPerMB\[2\] = \{([0-9.]+)f, ([0-9.]+)f\}", text)[0]]
     table["split"] = {"bf16": {"fixed_us": fx[0], "us_per_mb": pm[0]}, "int8": {"fixed_us": fx[1], "us_per_mb": pm[1]}}
+    table["mem_weight"] = float(re.findall(r"kMemWeight = ([0-9.]+);", text)[0])
     return table
 
 
