@@ -809,6 +809,17 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   p.out_bits = out_bits;
   p.out_shift = shift;
   p.q_img = ws;
+  // Split-K into int32 C by TMA reductions where C's base, pitch and row
+  // ends allow TMA (rows ending on a 16-byte boundary: a clipped TMA
+  // reduction would touch the rest of the row's last 16-byte piece), else
+  // by element-wise atomic adds.
+  CUtensorMap tc = tp;
+  p.c_tma = 0;
+  if (add_into_c && overrides().tma_store && aligned16(C) && (ldc * 4) % 16 == 0 && (N * 4) % 16 == 0) {
+    if (!encode_out(&tc, CU_TENSOR_MAP_DATA_TYPE_INT32, 4, C, (uint64_t)N, (uint64_t)M, (uint64_t)ldc, 1))
+      return true;
+    p.c_tma = 1;
+  }
   const int64_t units = tiles * splits;
   const int grid = (int)(units < d.sms ? units : d.sms);
   if (ovr.debug)
@@ -819,7 +830,7 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   const bool prof = g_prof_start && g_prof_stop;
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return true;
   g_launches.fetch_add(1);
-  if (launch_s8tm(qn, p_kmajor, tp, p, grid, st) != cudaSuccess) return true;
+  if (launch_s8tm(qn, p_kmajor, tp, tc, p, grid, st) != cudaSuccess) return true;
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return true;
   if (splits > 1 && !add_into_c) {
     g_launches.fetch_add(1);

@@ -87,6 +87,7 @@ struct S8tmParams {
   int splits, kb_per_split;
   int slab_kb;       // k-blocks per exact fp32 slab (1024 / kS8tmKB)
   int add_into_c;    // splits add their exact sums into C (int32, zeroed by the Q staging launch)
+  int c_tma;         // ... with TMA reductions through tmC (else element by element)
   int swap;
   void *C;
   int64_t ldc;
@@ -110,8 +111,9 @@ cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64
 // contiguous (boxes of 128 k x 128 rows); otherwise P's rows are the
 // contiguous dimension of its storage (boxes of 128 rows x 128 k, read
 // transposed by the converters).
-cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const S8tmParams &p, int grid,
-                        cudaStream_t st);
+// tc maps int32 C (32 x 32 boxes, 128-byte swizzle) when p.c_tma is set.
+cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const CUtensorMap &tc, const S8tmParams &p,
+                        int grid, cudaStream_t st);
 
 // Auxiliary kernels (aux_kernels.cu).  Each returns the launch error.
 // int8 -> bf16 (exact) of two matrices (A and B) in one launch; each is

@@ -79,7 +79,10 @@ struct S8tmCfg {
   static constexpr uint32_t kQBytes = 2 * kQHalf;      // the k-block's Q image
   static constexpr uint32_t kPOffset = 0;
   static constexpr uint32_t kQOffset = SP * kPBytes;  // 1024-byte aligned
-  static constexpr uint32_t kBarOffset = kQOffset + SQ * kQBytes;
+  // one 32 x 32 int32 block per epilogue warp, staging the TMA reductions
+  // of split-K into C (128-byte swizzle; 1024-byte aligned)
+  static constexpr uint32_t kEpiOffset = kQOffset + SQ * kQBytes;
+  static constexpr uint32_t kBarOffset = kEpiOffset + kEpiWarps * 4096;
   static constexpr uint32_t kNumBars = 2 * SP + 2 * SQ + 2 * NA + 5;
   static constexpr uint32_t kSmemBytes = kBarOffset + kNumBars * 8 + 16 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA is 227 KB");
@@ -115,7 +118,8 @@ __device__ __forceinline__ void store_row(const S8tmParams &p, const int32_t (&a
   const int64_t nq = p.Q_rows - q0;  // valid elements (>= 1)
   if (p.add_into_c) {
     // int32 C, zeroed by the Q staging kernel: every split adds its exact
-    // partial sums (integer addition, so any order gives the same C)
+    // partial sums (integer addition, so any order gives the same C), here
+    // element by element where C's alignment rules out TMA reductions
     int32_t *dst = reinterpret_cast<int32_t *>(p.C) + off0;
 #pragma unroll
     for (int i = 0; i < QN; ++i)
@@ -139,9 +143,47 @@ __device__ __forceinline__ void store_row(const S8tmParams &p, const int32_t (&a
   }
 }
 
+// Split-K of int32 C with TMA reductions: the warp's QN sums of its 32 P
+// rows, 32 Q columns at a time, staged as a 32 x 32 block (128-byte rows,
+// 16-byte chunk j of row r at chunk j ^ (r % 8)) and added into C by one TMA
+// reduction (element-wise atomic; the TMA clips a block that crosses C's
+// edges, and a block that starts outside C is not issued).  C[q][prow]
+// (swap): block row = q, column = lane; else C[prow][q]: row = lane.
+template <int QN>
+__device__ __forceinline__ void reduce_rows_tma(const CUtensorMap *tm, uint32_t buf, int lane, const int32_t (&acc)[QN],
+                                                bool swap, int32_t prow0, int32_t q0, int32_t P_rows, int32_t Q_rows) {
+#pragma unroll
+  for (int c = 0; c < QN / 32; ++c) {
+    if (lane == 0) bulk_wait_read_all();  // the previous reduction has read the block
+    __syncwarp();
+    if (swap) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        st_shared_u32(buf + i * 128 + ((((uint32_t)lane >> 2) ^ ((uint32_t)i & 7u)) << 4) + ((uint32_t)lane & 3u) * 4,
+                      static_cast<uint32_t>(acc[c * 32 + i]));
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        st_shared_v4(buf + lane * 128 + (((uint32_t)j ^ ((uint32_t)lane & 7u)) << 4),
+                     static_cast<uint32_t>(acc[c * 32 + 4 * j]), static_cast<uint32_t>(acc[c * 32 + 4 * j + 1]),
+                     static_cast<uint32_t>(acc[c * 32 + 4 * j + 2]), static_cast<uint32_t>(acc[c * 32 + 4 * j + 3]));
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0 && prow0 < P_rows && q0 + c * 32 < Q_rows) {
+      if (swap)
+        tma_reduce_add_2d(tm, buf, prow0, q0 + c * 32);
+      else
+        tma_reduce_add_2d(tm, buf, q0 + c * 32, prow0);
+      bulk_commit();
+    }
+  }
+}
+
 template <int QN, int SP, int SQ, int NA, bool PK>
 __global__ void __launch_bounds__(kThreadsS8tm, 1)
-    gemm_s8tm_kernel(const __grid_constant__ CUtensorMap tmP, const S8tmParams p) {
+    gemm_s8tm_kernel(const __grid_constant__ CUtensorMap tmP, const __grid_constant__ CUtensorMap tmC,
+                     const S8tmParams p) {
   using Cfg = S8tmCfg<QN, SP, SQ, NA>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -188,6 +230,7 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
     *abort_flag = 0u;
     fence_mbar_init();
     tma_prefetch_desc(&tmP);
+    if (p.c_tma) tma_prefetch_desc(&tmC);
   }
   if (warp == 1) tmem_alloc<Cfg::kTmemCols>(smem_addr(tmem_slot));
   tc_fence_before_sync();
@@ -399,9 +442,14 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
         ++acc_cnt;
       }
       if (!ok) break;
+      const int64_t q0 = (int64_t)w.tq * QN;
+      if (p.add_into_c && p.c_tma) {  // the whole warp: rows past the matrix are clipped by the TMA
+        reduce_rows_tma<QN>(&tmC, base + Cfg::kEpiOffset + (warp - 2) * 4096, lane, acc, p.swap != 0,
+                            w.tp * kBM + quad * 32, (int32_t)q0, p.P_rows, p.Q_rows);
+        continue;
+      }
       const int64_t prow = (int64_t)w.tp * kBM + r;
       if (prow >= p.P_rows) continue;
-      const int64_t q0 = (int64_t)w.tq * QN;
       // partials (split-K of int16 / int8 outputs) have row pitch N; C has ldc
       const int64_t ld = (p.splits > 1 && p.out_bits != 32) ? (int64_t)p.N : p.ldc;
       if (p.swap)  // C[q][prow]: per element the warp's lanes store 32 consecutive columns
@@ -411,6 +459,8 @@ __global__ void __launch_bounds__(kThreadsS8tm, 1)
     }
   }
 
+  // the epilogue's TMA reductions have completed before the CTA leaves
+  if (p.c_tma && warp >= 2 && warp < 2 + kEpiWarps && lane == 0) bulk_wait_all();
   griddep_launch_dependents();  // e.g. the split-K reduction may start setting up
   __syncwarp();
   tc_fence_before_sync();
@@ -432,7 +482,7 @@ __global__ void __launch_bounds__(256)
                         int64_t c_rows, int64_t c_cols, int64_t ldc) {
   griddep_launch_dependents();  // the GEMM waits for completion before reading
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= chunks) {  // the remaining threads zero C (int32, splits added by atomic adds)
+  if (t >= chunks) {  // the remaining threads zero C (int32, the splits' sums are added into it)
     if (!zero_c) return;
     // four consecutive elements of a row per step, with one 16-byte store
     // when the row pitch and base allow it
@@ -477,12 +527,13 @@ __global__ void __launch_bounds__(256)
 }
 
 template <int QN, int SP, int SQ, int NA, bool PK>
-cudaError_t launch_one(const CUtensorMap &tp, const S8tmParams &p, int grid, cudaStream_t st) {
+cudaError_t launch_one(const CUtensorMap &tp, const CUtensorMap &tc, const S8tmParams &p, int grid,
+                       cudaStream_t st) {
   using Cfg = S8tmCfg<QN, SP, SQ, NA>;
   auto kern = gemm_s8tm_kernel<QN, SP, SQ, NA, PK>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmemBytes);
   if (e != cudaSuccess) return e;
-  return launch_ex(kern, dim3(grid), dim3(kThreadsS8tm), Cfg::kSmemBytes, st, 1, tp, p);
+  return launch_ex(kern, dim3(grid), dim3(kThreadsS8tm), Cfg::kSmemBytes, st, 1, tp, tc, p);
 }
 
 }  // namespace
@@ -508,13 +559,15 @@ cudaError_t launch_s8tm_stage_q(const int8_t *src, int64_t sq, int64_t sk, int64
   return cudaGetLastError();
 }
 
-cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const S8tmParams &p, int grid,
-                        cudaStream_t st) {
+cudaError_t launch_s8tm(int qn, bool p_kmajor, const CUtensorMap &tp, const CUtensorMap &tc, const S8tmParams &p,
+                        int grid, cudaStream_t st) {
   // P stages x 16 KB + Q stages x (QN x 256 bytes): 9 x 16 + 2 x 32 KB
-  // (QN 128) or 10 x 16 + 3 x 16 KB (QN 64)
+  // (QN 128) or 10 x 16 + 3 x 16 KB (QN 64), and four 4 KB epilogue blocks
   if (qn == 128)
-    return p_kmajor ? launch_one<128, 9, 2, 4, true>(tp, p, grid, st) : launch_one<128, 9, 2, 4, false>(tp, p, grid, st);
-  return p_kmajor ? launch_one<64, 10, 3, 4, true>(tp, p, grid, st) : launch_one<64, 10, 3, 4, false>(tp, p, grid, st);
+    return p_kmajor ? launch_one<128, 9, 2, 4, true>(tp, tc, p, grid, st)
+                    : launch_one<128, 9, 2, 4, false>(tp, tc, p, grid, st);
+  return p_kmajor ? launch_one<64, 10, 3, 4, true>(tp, tc, p, grid, st)
+                  : launch_one<64, 10, 3, 4, false>(tp, tc, p, grid, st);
 }
 
 }  // namespace gb300
