@@ -583,3 +583,21 @@ def test_int8_converted_in_kernel_split_into_padded_c(M, N, K, layout, splits, m
     A, B = _inputs("int8", M, N, K, layout, seed=M + K)
     C = U.run("int8", A, B, layout, ldc=N + 5, c_off=3)
     _check("int8", A, B, layout, C)
+
+
+@pytest.mark.parametrize("M,N,K,layout", [(16, 512, 4096, COL), (100, 1008, 3000, ROW), (1000, 64, 3008, ROW),
+                                          (300, 128, 4096, COL), (9, 144, 1024, ROW)],
+                         ids=["swap", "swap-transposed", "direct", "direct-Bcol", "swap-small"])
+@pytest.mark.parametrize("ldc_pad", [0, 4, 12])
+def test_int8_converted_in_kernel_split_tma_reduction(M, N, K, layout, ldc_pad, monkeypatch):
+    """Split-K of int32 outputs on the small-operand path where C allows TMA
+    (16-byte aligned base and pitch, rows ending on a 16-byte boundary):
+    the splits' sums go into C by TMA tensor reductions, clipped at the
+    matrix edges (ragged tiles, padded pitch untouched), bit-exact and equal
+    to the element-wise atomic adds (GB300_GEMM_TMA_STORE=0)."""
+    monkeypatch.setenv("GB300_GEMM_SPLITS", "3")
+    A, B = _inputs("int8", M, N, K, layout, seed=M + N + ldc_pad)
+    C = U.run("int8", A, B, layout, ldc=N + ldc_pad)
+    _check("int8", A, B, layout, C)
+    monkeypatch.setenv("GB300_GEMM_TMA_STORE", "0")
+    assert np.array_equal(U.run("int8", A, B, layout, ldc=N + ldc_pad), C)
