@@ -392,6 +392,28 @@ __device__ __forceinline__ void tma_out_narrow(const CUtensorMap *tm, uint32_t b
   }
 }
 
+// One 32-column chunk of a lane's int32 sums (row `row`, columns x ..): to
+// C (int32, or requantised) or to the split's partials (wrow), through the
+// warp's TMA staging block when out_tma says so (the warp's rows y0 ..),
+// else directly.
+__device__ __forceinline__ void store_s32_chunk(const TcParams &p, const CUtensorMap *tm, uint32_t ebuf, int lane,
+                                                int out_tma, const uint32_t (&v)[32], int x, int y0, int split,
+                                                bool row_ok, int64_t row, uint32_t *wrow, bool ws_vec) {
+  if (out_tma != kOutDirect) {
+    if (out_tma == kOutTmaWs)
+      tma_out_words32<true>(tm, ebuf, lane, v, x, y0, split, y0 < p.M && x < p.N);
+    else if (p.out_bits == 32)
+      tma_out_words32<false>(tm, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+    else
+      tma_out_narrow(tm, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
+  } else if (row_ok) {
+    if (wrow)
+      store_words<32>(wrow, x, p.N, ws_vec, v);
+    else
+      store_s8_result<32>(p, row, x, v);
+  }
+}
+
 template <int W>
 __device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
   if constexpr (W == 32)
@@ -554,6 +576,47 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
       const int col0 = w.tn * BN + colpart * CPT;
       const int y0 = w.tm * kBM + quad * 32;  // first row of this warp's blocks
       if constexpr (EPI == kEpiS32) {
+        if (w.kb1 - w.kb0 <= p.slab_kb) {
+          // One slab (K of the unit <= 1024): its exact fp32 sums are the
+          // result, streamed 32 columns at a time as in the bf16 epilogue
+          // instead of being gathered into int32 registers.
+          const uint32_t b = acc_cnt & 1u, aph = (acc_cnt >> 1) & 1u;
+          if (!__all_sync(0xffffffffu, mbar_wait(accf_bar(b), aph, abort_flag, p.err, p.wait_limit_ns))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+          const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
+          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+                                 : nullptr;
+#pragma unroll 1
+          for (int c = 0; c < CPT / 32; ++c) {
+            uint32_t v[32];
+            tmem_ld<32>(t0 + c * 32, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(__float2int_rn(__uint_as_float(v[i])));
+            store_s32_chunk(p, &tmOut, ebuf, lane, out_tma, v, col0 + c * 32, y0, w.split, row_ok, row, wrow, ws_vec);
+          }
+          if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
+            constexpr int kTail = (CPT / 32) * 32;
+            uint32_t v[16];
+            tmem_ld<16>(t0 + kTail, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(__float2int_rn(__uint_as_float(v[i])));
+            if (row_ok) {
+              if (split)
+                store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+              else
+                store_s8_result<16>(p, row, col0 + kTail, v);
+            }
+          }
+          tc_fence_before_sync();
+          mbar_arrive(acce_bar(b));
+          ++acc_cnt;
+          continue;
+        }
         int32_t acc[CPT];
 #pragma unroll
         for (int i = 0; i < CPT; ++i) acc[i] = 0;
