@@ -42,7 +42,9 @@
  *     benchmarks (int8 results are identical either way; bf16 results may
  *     differ in summation order, within the same accuracy): GB300_GEMM_BN,
  *     GB300_GEMM_PAIR, GB300_GEMM_SPLITS, GB300_GEMM_SKINNY_MAX_M,
- *     GB300_GEMM_TMA_STORE=0, GB300_GEMM_PDL=0, GB300_GEMM_S8TM=0 (int8
+ *     GB300_GEMM_TMA_STORE=0 (results stored, and split-K sums added into
+ *     C, element by element instead of by TMA), GB300_GEMM_PDL=0 (plain
+ *     stream ordering between the library's kernels), GB300_GEMM_S8TM=0 (int8
  *     GEMMs with one operand of at most 128 rows take the general path
  *     instead of converting the large operand inside the kernel),
  *     GB300_GEMM_TINY_MAX_MACS (largest M*N*K of an int8 GEMM computed in one

@@ -73,7 +73,8 @@ namespace {
 // GB300_GEMM_BN (128, 192, 224 or 256) forces the tile width,
 // GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
 // split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
-// CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores, GB300_GEMM_PDL=0
+// CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores (and scalar atomic
+// adds for the small-operand kernel's split-K), GB300_GEMM_PDL=0
 // plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
 // small-operand shapes, GB300_GEMM_TINY_MAX_MACS the largest
 // int8 problem (M * N * K) sent to the one-launch CUDA-core kernel (0
