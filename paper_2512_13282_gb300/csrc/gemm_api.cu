@@ -712,16 +712,43 @@ bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t inner, uint64_t
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// K splits of the small-operand int8 kernel: enough units to give every SM
-// one, at least 4 k-blocks (of 128) per split, at most 16 (or the forced
-// count); rounded so that no split is empty.
-int64_t s8tm_splits(int64_t tiles, int64_t num_kb, int sms, int forced) {
-  int64_t splits = (int64_t)sms / tiles;
-  if (splits > num_kb / 4) splits = num_kb / 4;
-  if (splits > 16) splits = 16;
-  if (splits < 1) splits = 1;
-  if (forced >= 1) splits = forced < num_kb ? forced : num_kb;
-  return ceil_div(num_kb, ceil_div(num_kb, splits));
+// K splits of the small-operand int8 kernel.  A unit (one P tile, one
+// split) is a chain of k-blocks that each pass the converter, the TMEM store
+// and the MMA in turn, ~0.57 us a k-block on GB300 whatever the bytes, and
+// the CTAs (one per SM) run their units one after the other; so the split
+// minimises rounds * (k-blocks per unit + kS8tmUnitKb), the per-unit start
+// and drain counted in k-blocks, plus kS8tmReduceKb when int16 / int8
+// outputs need the reduction launch.  Measured on GB300 (whole GEMM after a
+// 512 MiB flush), this picks the fastest of 1-8 splits for int32 outputs on
+// 128 x 11008 x 4096 (3 splits: 258 units in two rounds of 11 k-blocks,
+// 34.3 -> 30.2 us against one split on 86 SMs), 128 x 12288 x 4096,
+// 128 x 4096 x 11008, 128 x 4096 x 4096, 16 x 4096 x 4096 and
+// 8192 x 64 x 8192, and for int16 outputs on 128 x 11008 / 12288 x 4096
+// (one split: the reduction launch costs more than the shorter chains gain)
+// and 128 x 4096 x 4096 (4 splits).  At least 4 k-blocks (of 128) per split,
+// at most 16 splits (or the forced count); rounded so that no split is
+// empty.
+constexpr int64_t kS8tmUnitKb = 2;
+constexpr int64_t kS8tmReduceKb = 10;
+
+int64_t s8tm_splits(int64_t tiles, int64_t num_kb, int sms, int forced, bool reduce_launch) {
+  if (forced >= 1) {
+    const int64_t f = forced < num_kb ? forced : num_kb;
+    return ceil_div(num_kb, ceil_div(num_kb, f));
+  }
+  int64_t best = 1, best_cost = -1;
+  for (int64_t s = 1; s <= 16 && s <= num_kb; ++s) {
+    const int64_t kb_per = ceil_div(num_kb, s);
+    const int64_t s2 = ceil_div(num_kb, kb_per);
+    if (s2 != s || (s2 > 1 && kb_per < 4)) continue;  // a count already seen, or too short a split
+    const int64_t rounds = ceil_div(tiles * s2, (int64_t)sms);
+    const int64_t cost = rounds * (kb_per + kS8tmUnitKb) + (s2 > 1 && reduce_launch ? kS8tmReduceKb : 0);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = s2;
+    }
+  }
+  return best;
 }
 
 // Which operand the small-operand int8 kernel streams, if any: P = B with
@@ -766,7 +793,7 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   const int64_t num_kb = ceil_div(K, kS8tmKB);
   const int64_t tiles_p = ceil_div(P_rows, kBM), tiles_q = ceil_div(Q_rows, qn);
   const int64_t tiles = tiles_p * tiles_q;
-  int64_t splits = s8tm_splits(tiles, num_kb, d.sms, ovr.splits);
+  int64_t splits = s8tm_splits(tiles, num_kb, d.sms, ovr.splits, out_bits != 32);
   const int64_t kb_per = ceil_div(num_kb, splits);
   gemm_status_t s;
   // split-K: int32 outputs are added into C (zeroed by the staging launch),
@@ -1017,7 +1044,7 @@ gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_l
     const int64_t Q_rows = swap ? M : N, P_rows = swap ? N : M;
     const int qn = Q_rows <= 64 ? 64 : 128;
     const int64_t tiles = ceil_div(P_rows, kBM) * ceil_div(Q_rows, qn);
-    const int64_t splits = s8tm_splits(tiles, ceil_div(K, kS8tmKB), sms, overrides().splits);
+    const int64_t splits = s8tm_splits(tiles, ceil_div(K, kS8tmKB), sms, overrides().splits, false);
     out->route = GEMM_ROUTE_SMALL_OPERAND;
     out->bn = qn;
     out->splits = (int)splits;
