@@ -70,7 +70,8 @@ namespace {
 
 // Test and benchmark overrides of the planner, read from the environment
 // once (at the first call) and again by gemm_reload_overrides():
-// GB300_GEMM_BN (128, 192, 224 or 256) forces the tile width,
+// GB300_GEMM_BN (64, 96, 128, 192, 224 or 256; 64 and 96 for bf16 only)
+// forces the tile width,
 // GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
 // split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
 // CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores (and scalar atomic
@@ -372,7 +373,7 @@ struct Plan {
 // rule.
 double modelled_us(int64_t M, int64_t N, bool int8, bool pair, int bn, int64_t splits, int64_t kb_per,
                    int64_t rounds) {
-  const int wi = bn == 128 ? 0 : bn == 192 ? 1 : bn == 224 ? 2 : 3;
+  const int wi = bn == 64 ? 0 : bn == 96 ? 1 : bn == 128 ? 2 : bn == 192 ? 3 : bn == 224 ? 4 : 5;
   const plan_table::StepCost c = plan_table::kCost[int8 ? 1 : 0][pair ? 1 : 0][wi];
   double t = (double)rounds * ((double)kb_per * c.kstep_us + c.unit_us);
   if (splits > 1)
@@ -397,8 +398,11 @@ double dram_us(int64_t M, int64_t N, int64_t K, bool int8, bool pair) {
 
 Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms, int pairs) {
   Plan pl{};
-  static const int kWidthsKMajor[] = {256, 224, 192, 128};
-  static const int kWidthsMNMajor[] = {256, 192, 128};
+  // compiled widths, widest first: the bf16 single-CTA kernels also come 64
+  // and 96 wide (96 for B column-major only), for memory-bound GEMMs with
+  // few rows
+  static const int kWidthsKMajor[] = {256, 224, 192, 128, 96, 64};
+  static const int kWidthsMNMajor[] = {256, 192, 128, 64};
   static const int kPairWidthsMNMajor[] = {256, 128};
   const Overrides ovr = overrides();
   const bool int8 = epi == kEpiS32;
@@ -412,12 +416,13 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
     if (pair && (M <= kBM || pairs <= 0)) continue;  // the second CTA would only compute padding
     if (ovr.pair >= 0 && (ovr.pair != 0) != pair) continue;
     const int *widths = b_kmajor ? kWidthsKMajor : (pair ? kPairWidthsMNMajor : kWidthsMNMajor);
-    const int nw = b_kmajor ? 4 : (pair ? 2 : 3);
+    const bool narrow = !pair && !int8;
+    const int nw = b_kmajor ? (narrow ? 6 : 4) : (pair ? 2 : (narrow ? 4 : 3));
     const int64_t slots = pair ? pairs : sms;
     const int64_t tiles_m = ceil_div(M, pair ? 2 * kBM : kBM);
     for (int i = 0; i < nw; ++i) {
       const int bn = widths[i];
-      if (N <= 128 && bn != 128) continue;
+      if (N <= 128 && bn > 128) continue;
       if (ovr.bn > 0 && ovr.bn != bn) continue;
       const int64_t tiles = tiles_m * ceil_div(N, bn);
       int64_t seen[17] = {};

@@ -27,8 +27,12 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 // Tile widths compiled for the bf16 epilogue, with their stage counts and
 // output path (TMA stores through four 4 KB staging blocks, or, where those
 // would cost a pipeline stage, through four 1 KB blocks of 16 columns):
-// 128 (6, 4 KB), 192 (5, 4 KB), 224 (5, 1 KB; B column-major only), 256
-// (4, 4 KB) -- in each case the deepest ring that fits (tc_max_stages).
+// 64 (8, 4 KB), 96 (7, 4 KB; B column-major only), 128 (6, 4 KB), 192 (5,
+// 4 KB), 224 (5, 1 KB; B column-major only), 256 (4, 4 KB) -- in each case
+// the deepest ring that fits (tc_max_stages).  The narrow tiles serve
+// memory-bound GEMMs with few rows: N / 96 tiles of 128 x 96 fill the SMs
+// without a K split, and so without the reduction launch (bf16 128 x 11008
+// x 4096: 115 CTAs), and 64 fits N = 64 without padding columns.
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
@@ -37,12 +41,15 @@ cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUten
       case 224: return launch_one<224, tc_max_stages(224, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
       case 192: return launch_one<192, tc_max_stages(192, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
       case 128: return launch_one<128, tc_max_stages(128, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 96: return launch_one<96, tc_max_stages(96, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 64: return launch_one<64, tc_max_stages(64, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   } else {
     switch (v.bn) {
       case 256: return launch_one<256, tc_max_stages(256, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
       case 192: return launch_one<192, tc_max_stages(192, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
       case 128: return launch_one<128, tc_max_stages(128, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 64: return launch_one<64, tc_max_stages(64, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;

@@ -80,7 +80,11 @@ GB300 = {"sms": 152, "pair_slots": 76, "smem_per_cta": 232448, "tmem_cols": 512,
 BM = 128          # rows of C per CTA (MMA M)
 BK = 64           # K per pipeline stage: one 128-byte swizzle row of bf16
 KB_DEPTH = BK
-WIDTHS = (128, 192, 224, 256)
+WIDTHS = (64, 96, 128, 192, 224, 256)
+# the bf16 single-CTA kernels also come 64 and 96 wide (96 for B column-major
+# only): tiles for memory-bound GEMMs with few rows, which fill the SMs
+# without a K split; they do not meet Eq. 4 and are chosen only by time
+NARROW = (64, 96)
 
 
 class Variant:
@@ -138,10 +142,13 @@ def compiled_variants():
     gemm_tc2_*.cu): bf16 with one epilogue warpgroup; int8 with two for
     tiles wider than 128; 224 (and the pair's 192) for B column-major only;
     the bf16 224-wide kernels stage through 1 KB blocks; the int8 192/224
-    ones come with TMA staging blocks or with direct stores."""
-    v = []
+    ones come with TMA staging blocks or with direct stores; and the narrow
+    bf16 single-CTA tiles, 64 (both layouts) and 96 (B column-major)."""
+    v = [Variant("bf16", False, 64, False, 4, 1), Variant("bf16", False, 96, True, 4, 1)]
     for pair in (False, True):
         for bn in WIDTHS:
+            if bn in NARROW:
+                continue
             km_only = bn == 224 or (pair and bn == 192)
             v.append(Variant("bf16", pair, bn, km_only, 4, 2 if bn == 224 else 1))
             ew = 4 if bn == 128 else 8
@@ -181,11 +188,21 @@ def _ceil(a, b):
     return -(-a // b)
 
 
-def candidate_plans(M, N, K, b_kmajor, sms=None, pair_slots=None):
+def plan_widths(dtype, pair, b_kmajor):
+    """Tile widths compiled for one operand type, family and B layout, in
+    the planner's order (widest first)."""
+    if pair:
+        return (256, 224, 192, 128) if b_kmajor else (256, 128)
+    if b_kmajor:
+        return (256, 224, 192, 128, 96, 64) if dtype == "bf16" else (256, 224, 192, 128)
+    return (256, 192, 128, 64) if dtype == "bf16" else (256, 192, 128)
+
+
+def candidate_plans(M, N, K, dtype, b_kmajor, sms=None, pair_slots=None):
     """Every (family, BN, S) the planner considers for an M x N x K GEMM,
     with its tile count, K steps per unit and rounds.  Pairs need M > 128;
-    tiles narrower than the matrix only where N > 128; S keeps >= 4 K steps
-    per unit and at most 2 units per slot."""
+    tiles wider than 128 only where N > 128; S keeps >= 4 K steps per unit
+    and at most 2 units per slot."""
     sms = sms or GB300["sms"]
     pair_slots = pair_slots if pair_slots is not None else GB300["pair_slots"]
     num_kb = _ceil(K, BK)
@@ -194,10 +211,9 @@ def candidate_plans(M, N, K, b_kmajor, sms=None, pair_slots=None):
         if pair and (M <= BM or pair_slots <= 0):
             continue
         slots = pair_slots if pair else sms
-        widths = (256, 224, 192, 128) if b_kmajor else ((256, 128) if pair else (256, 192, 128))
         tiles_m = _ceil(M, 2 * BM if pair else BM)
-        for bn in widths:
-            if N <= 128 and bn != 128:
+        for bn in plan_widths(dtype, pair, b_kmajor):
+            if N <= 128 and bn > 128:
                 continue
             tiles = tiles_m * _ceil(N, bn)
             seen = set()
@@ -266,7 +282,7 @@ def choose_plan(M, N, K, dtype, b_kmajor, table, sms=None, pair_slots=None):
     """The planner: the candidate of least rank_us (the first one, in
     candidate order, on a tie)."""
     best, best_c = None, math.inf
-    for p in candidate_plans(M, N, K, b_kmajor, sms, pair_slots):
+    for p in candidate_plans(M, N, K, dtype, b_kmajor, sms, pair_slots):
         c = rank_us(M, N, K, dtype, p, table)
         if c < best_c - 1e-9:
             best, best_c = p, c
@@ -389,7 +405,7 @@ def balanced_search(M, N, K, dtype, b_kmajor, measure, table, sms=None, pair_slo
     BN, S) by modelled time; the steps measure them in that order --
     `measure(plan)` returns the measured time -- until the first measured
     slowdown.  Returns (best plan measured, its time, plans measured)."""
-    cands = candidate_plans(M, N, K, b_kmajor, sms, pair_slots)
+    cands = candidate_plans(M, N, K, dtype, b_kmajor, sms, pair_slots)
     cands.sort(key=lambda q: plan_cost_us(M, N, K, dtype, q, table))
     best, best_t, prev, n = None, math.inf, math.inf, 0
     for p in cands:
@@ -427,8 +443,8 @@ def header_text(table, source="plan_measurements.json"):
         "  float unit_us;   // per unit: start, accumulator drain, stores",
         "};",
         "",
-        "// [0 bf16, 1 int8][0 single CTA, 1 CTA pair][BN 128, 192, 224, 256]",
-        "constexpr StepCost kCost[2][2][4] = {",
+        "// [0 bf16, 1 int8][0 single CTA, 1 CTA pair][BN %s]; {0, 0}: not compiled" % ", ".join(map(str, WIDTHS)),
+        "constexpr StepCost kCost[2][2][%d] = {" % len(WIDTHS),
     ]
     for dtype in ("bf16", "int8"):
         lines.append("    {")

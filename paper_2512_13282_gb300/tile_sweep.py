@@ -6,10 +6,13 @@ each shape of a fixed set -- the tensor-core GEMMs of the benchmark
 workloads and a seeded sample of the roofline sweep sizes -- every plan the
 library can be forced into (kernel family: one CTA per 128-row tile or a CTA
 pair per 256-row tile; tile width BN; split-K factor S) is timed with CUDA
-events after a 512 MiB L2 flush, median of `reps`.  The result is written as
-JSON; tile_model.py fits the planner's cost table to it.
+events after a 512 MiB L2 flush: the mean of `reps` launches without the
+fastest and the slowest (the event clock advances in steps of about 1 us on
+GB300, so a median of a few launches of a 10-30 us GEMM is off by up to a
+step; a mean of many is not).  The result is written as JSON; tile_model.py
+fits the planner's cost table to it.
 
-    python -m paper_2512_13282_gb300.tile_sweep OUT.json [--reps 5] [--sample 40]
+    python -m paper_2512_13282_gb300.tile_sweep OUT.json [--reps 15] [--sample 40]
 
 Needs a GPU and the built library.  Results of int8 GEMMs are exact whatever
 the plan, and bf16 results differ only in summation order, so no plan is
@@ -69,7 +72,7 @@ def main(argv=None):
 
     ap = argparse.ArgumentParser()
     ap.add_argument("out")
-    ap.add_argument("--reps", type=int, default=5)
+    ap.add_argument("--reps", type=int, default=15)
     ap.add_argument("--sample", type=int, default=40)
     args = ap.parse_args(argv)
     Bld.build()
@@ -112,7 +115,8 @@ def main(argv=None):
             if r >= 2:
                 ts.append((a, b))
         torch.cuda.synchronize()
-        return statistics.median(x.elapsed_time(y) * 1e3 for x, y in ts)
+        us = sorted(x.elapsed_time(y) * 1e3 for x, y in ts)
+        return statistics.mean(us[1:-1]) if len(us) > 2 else statistics.mean(us)
 
     rows = []
     t0 = time.time()
@@ -120,7 +124,7 @@ def main(argv=None):
         setenv(TC_ONLY)
         default_us = time_plan(M, N, K, dtype, layout)
         plans = []
-        for c in candidate_plans(M, N, K, layout == W.B_COL_MAJOR, sms=sms, pair_slots=GB300["pair_slots"]):
+        for c in candidate_plans(M, N, K, dtype, layout == W.B_COL_MAJOR, sms=sms, pair_slots=GB300["pair_slots"]):
             setenv(dict(TC_ONLY, GB300_GEMM_PAIR=int(c["pair"]), GB300_GEMM_BN=c["bn"],
                         GB300_GEMM_SPLITS=c["splits"]))
             plans.append(dict(c, us=round(time_plan(M, N, K, dtype, layout), 3)))
@@ -133,7 +137,8 @@ def main(argv=None):
     setenv({})
     with open(args.out, "w") as f:
         json.dump({"device": torch.cuda.get_device_name(dev), "sms": sms, "reps": args.reps,
-                   "flush": "512 MiB write before every launch", "seconds": round(time.time() - t0, 1),
+                   "flush": "512 MiB write before every launch", "statistic": "mean without min and max",
+                   "seconds": round(time.time() - t0, 1),
                    "shapes": rows}, f, indent=0)
 
 

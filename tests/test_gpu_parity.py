@@ -334,6 +334,27 @@ def test_parity_every_tile_width(dtype, layout, bn, pair, monkeypatch):
         _check(dtype, A, B, layout, C)
 
 
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("bn", [64, 96])
+def test_parity_narrow_bf16_tiles(layout, bn, monkeypatch):
+    """The 64- and 96-wide bf16 kernels (96 for B column-major only) on
+    ragged multi-tile shapes, N narrower than one tile, few rows and long K,
+    with and without split-K; the plan query reports the forced width."""
+    if layout == ROW and bn == 96:
+        pytest.skip("no 96-wide tile for row-major B")
+    monkeypatch.setenv("GB300_GEMM_BN", str(bn))
+    monkeypatch.setenv("GB300_GEMM_PAIR", "0")
+    for (M, N, K, splits) in ((300, 700, 1500, "1"), (130, 450, 3000, "3"), (128, 1100, 2048, "1"),
+                              (1000, 64, 4100, "2"), (129, 97, 333, "1"), (40, 200, 5000, "4")):
+        monkeypatch.setenv("GB300_GEMM_SPLITS", splits)
+        G.gemm_reload_overrides()
+        st, plan = G.gemm_plan_query(M, N, K, False, layout)
+        assert st == 0 and plan["route"] == G.GEMM_ROUTE_TC_SINGLE and plan["bn"] == bn, plan
+        A, B = _inputs("bf16", M, N, K, layout, seed=bn + M + N)
+        C = U.run("bf16", A, B, layout)
+        _check("bf16", A, B, layout, C)
+
+
 SKINNY = [(1, 1, 1), (1, 11008, 4096), (2, 257, 777), (3, 1000, 4100), (5, 300, 64), (8, 4096, 4096),
           (13, 555, 2049), (16, 4096, 4096), (16, 96, 20000)]
 

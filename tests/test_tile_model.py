@@ -44,22 +44,37 @@ def test_single_core_ip_prefers_the_largest_tile_that_fits():
 
 
 def test_every_compiled_variant_satisfies_eq4_and_eq5():
+    """Eq. 5 (the ring fits) for every compiled kernel, Eq. 4 (a stage's
+    MMA time covers its TMA fill) for all but the narrow bf16 tiles, which
+    exist for memory-bound GEMMs and are chosen only by measured time."""
     for v in T.compiled_variants():
         comp, comm = v.eq4_cycles()
-        assert comp >= comm, v
+        assert (comp >= comm) == (v.bn not in T.NARROW), v
         s = v.max_stages()
         assert s >= 2 and v.smem_bytes(s) <= T.GB300["smem_per_cta"] < v.smem_bytes(s + 1), v
         assert v.tmem_cols() <= T.GB300["tmem_cols"], v
 
 
+def test_planner_widths_are_the_compiled_variants():
+    """The widths the planner may pick per operand type, family and B
+    layout are exactly the compiled kernels."""
+    compiled = {(v.dtype, v.pair, v.bn, km) for v in T.compiled_variants() for km in (True, False)
+                if km or not v.kmajor_only}
+    planned = {(d, pair, bn, km) for d in ("bf16", "int8") for pair in (False, True) for km in (True, False)
+               for bn in T.plan_widths(d, pair, km)}
+    assert planned == compiled
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "int8"])
 @pytest.mark.parametrize("pair", [False, True], ids=["single", "pair"])
-@pytest.mark.parametrize("bn", [128, 192, 224, 256])
+@pytest.mark.parametrize("bn", [64, 96, 128, 192, 224, 256])
 def test_library_pipeline_depths_are_the_model_maximum(lib, monkeypatch, dtype, pair, bn):
     """The stage count the library compiles for each variant equals Eq. 5's
     maximum (the C++ derives it from the same budget)."""
+    if bn in T.NARROW and (dtype != "bf16" or pair):
+        pytest.skip("the narrow tiles are bf16 single-CTA kernels")
     for K, kmajor in ((4096, True), (16384, True), (4096, False)):
-        if not kmajor and (bn == 224 or (pair and bn == 192)):
+        if bn not in T.plan_widths(dtype, pair, kmajor):
             continue
         monkeypatch.setenv("GB300_GEMM_BN", str(bn))
         monkeypatch.setenv("GB300_GEMM_PAIR", "1" if pair else "0")
