@@ -719,8 +719,9 @@ bool encode_s8_rows(CUtensorMap *map, const void *base, uint64_t inner, uint64_t
 
 // K splits of the small-operand int8 kernel.  A unit (one P tile, one
 // split) is a chain of k-blocks that each pass the converter, the TMEM store
-// and the MMA in turn, ~0.57 us a k-block on GB300 whatever the bytes, and
-// the CTAs (one per SM) run their units one after the other; so the split
+// and the MMA in turn, ~0.57 us a k-block on GB300 until every SM streams
+// (then the P stream's rate takes over), and the CTAs (one per SM) run
+// their units one after the other; so the split
 // minimises rounds * (k-blocks per unit + kS8tmUnitKb), the per-unit start
 // and drain counted in k-blocks, plus kS8tmReduceKb when int16 / int8
 // outputs need the reduction launch.  Measured on GB300 (whole GEMM after a
