@@ -41,7 +41,9 @@
  *   - Environment variables that override the planner, for tests and
  *     benchmarks (int8 results are identical either way; bf16 results may
  *     differ in summation order, within the same accuracy): GB300_GEMM_BN,
- *     GB300_GEMM_PAIR, GB300_GEMM_SPLITS, GB300_GEMM_SKINNY_MAX_M,
+ *     GB300_GEMM_PAIR, GB300_GEMM_SPLITS, GB300_GEMM_TAIL_SPLITS (0: no
+ *     split tail; S >= 2: split the last round's tiles in S where the plan
+ *     has such a round), GB300_GEMM_SKINNY_MAX_M,
  *     GB300_GEMM_TMA_STORE=0 (results stored, and split-K sums added into
  *     C, element by element instead of by TMA), GB300_GEMM_PDL=0 (plain
  *     stream ordering between the library's kernels), GB300_GEMM_S8TM=0 (int8
@@ -240,7 +242,10 @@ gemm_status_t gemm_selftest_wait_timeout(uint64_t limit_ns, gemm_stream_t stream
  *   and ldc = N or K) and 16-byte aligned; the planner overrides in force
  *   (GB300_GEMM_*) apply.
  *   out->route: GEMM_ROUTE_*; bn: tile width (the small operand's tile
- *   height for GEMM_ROUTE_SMALL_OPERAND); splits: K split factor; stages:
+ *   height for GEMM_ROUTE_SMALL_OPERAND); splits: K split factor;
+ *   tail_splits: 0, or the split of the tiles of the last, partly filled
+ *   round of the tensor-core kernel (each in tail_splits K ranges, summed
+ *   by the split-K reduction over those tiles only); stages:
  *   pipeline depth of the tensor-core kernel; grid: CTAs launched;
  *   model_us: modelled time of the tensor-core kernel and split-K reduction
  *   (the quantity the planner minimises); dram_us: the DRAM time of the
@@ -264,6 +269,7 @@ typedef struct {
   int grid;
   double model_us;
   double dram_us;
+  int tail_splits;
 } gemm_plan_t;
 gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_layout, int sms, int pair_slots,
                               gemm_plan_t *out);

@@ -202,6 +202,28 @@ __device__ __forceinline__ Piece piece_of(uint64_t t, uint32_t cpr, int64_t N) {
   return pc;
 }
 
+// Piece t of the part of C that rt covers; false when it lies outside C.
+__device__ __forceinline__ bool reduce_piece(uint64_t t, uint32_t cpr, int64_t M, int64_t N, const ReduceTiles &rt,
+                                             Piece *pc) {
+  if (rt.count == 0) {
+    if (t >= (uint64_t)M * cpr) return false;
+    *pc = piece_of(t, cpr, N);
+    return true;
+  }
+  const uint32_t cpt = (uint32_t)rt.cols / 4;
+  const uint64_t per_tile = (uint64_t)rt.rows * cpt;
+  if (t >= per_tile * (uint64_t)rt.count) return false;
+  const int ti = (int)(t / per_tile);
+  const uint32_t rem = (uint32_t)(t - (uint64_t)ti * per_tile);
+  int tm, tn;
+  raster_tile(rt.first + ti, rt.tiles_m, rt.tiles_n, rt.group_m, &tm, &tn);
+  pc->r = (int64_t)tm * rt.rows + rem / cpt;
+  pc->c = (int64_t)tn * rt.cols + (int64_t)(rem % cpt) * 4;
+  if (pc->r >= M || pc->c >= N) return false;
+  pc->n = N - pc->c < 4 ? (int)(N - pc->c) : 4;
+  return true;
+}
+
 template <typename T>
 __device__ __forceinline__ void sum_piece(const T *__restrict__ ws, int splits, int64_t MN, int64_t N,
                                           const Piece &pc, T (&v)[4]) {
@@ -224,11 +246,11 @@ __device__ __forceinline__ void sum_piece(const T *__restrict__ ws, int splits, 
 
 __global__ void __launch_bounds__(kThreads)
     splitk_reduce_bf16_kernel(const float *__restrict__ ws, int splits, int64_t M, int64_t N,
-                              uint16_t *__restrict__ C, int64_t ldc, uint32_t cpr) {
+                              uint16_t *__restrict__ C, int64_t ldc, uint32_t cpr, const ReduceTiles rt) {
   griddep_wait();  // the partials come from the GEMM launched just before
   const uint64_t t = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (uint64_t)M * cpr) return;
-  const Piece pc = piece_of(t, cpr, N);
+  Piece pc;
+  if (!reduce_piece(t, cpr, M, N, rt, &pc)) return;
   float v[4];
   sum_piece(ws, splits, M * N, N, pc, v);
   uint16_t *dst = C + pc.r * ldc + pc.c;
@@ -248,11 +270,11 @@ __global__ void __launch_bounds__(kThreads)
 // int32 partials; stored as int32, or requantised to int16 / int8.
 __global__ void __launch_bounds__(kThreads)
     splitk_reduce_s32_kernel(const int32_t *__restrict__ ws, int splits, int64_t M, int64_t N, void *__restrict__ C,
-                             int64_t ldc, int out_bits, int shift, uint32_t cpr) {
+                             int64_t ldc, int out_bits, int shift, uint32_t cpr, const ReduceTiles rt) {
   griddep_wait();
   const uint64_t t = (uint64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (uint64_t)M * cpr) return;
-  const Piece pc = piece_of(t, cpr, N);
+  Piece pc;
+  if (!reduce_piece(t, cpr, M, N, rt, &pc)) return;
   int32_t v[4];
   sum_piece(ws, splits, M * N, N, pc, v);
   if (out_bits == 32) {
@@ -375,20 +397,26 @@ cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esi
   return cudaGetLastError();
 }
 
+// Pieces (4 elements of a row) the reduction covers.
+static uint64_t reduce_items(int64_t M, uint32_t cpr, const ReduceTiles &rt) {
+  return rt.count == 0 ? (uint64_t)M * cpr : (uint64_t)rt.count * rt.rows * ((uint32_t)rt.cols / 4);
+}
+
 cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, int64_t N,
-                                      uint16_t *C, int64_t ldc, int sms, cudaStream_t st) {
-  (void)sms;
-  const uint64_t cpr = (uint64_t)(N + 3) / 4, items = (uint64_t)M * cpr;
+                                      uint16_t *C, int64_t ldc, const ReduceTiles &rt, cudaStream_t st) {
+  const uint32_t cpr = (uint32_t)((N + 3) / 4);
+  const uint64_t items = reduce_items(M, cpr, rt);
   return launch_ex(splitk_reduce_bf16_kernel, dim3((unsigned)((items + kThreads - 1) / kThreads)), dim3(kThreads),
-                   0, st, 1, ws, splits, M, N, C, ldc, (uint32_t)cpr);
+                   0, st, 1, ws, splits, M, N, C, ldc, cpr, rt);
 }
 
 cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N, void *C,
-                                     int64_t ldc, int out_bits, int shift, int sms, cudaStream_t st) {
-  (void)sms;
-  const uint64_t cpr = (uint64_t)(N + 3) / 4, items = (uint64_t)M * cpr;
+                                     int64_t ldc, int out_bits, int shift, const ReduceTiles &rt,
+                                     cudaStream_t st) {
+  const uint32_t cpr = (uint32_t)((N + 3) / 4);
+  const uint64_t items = reduce_items(M, cpr, rt);
   return launch_ex(splitk_reduce_s32_kernel, dim3((unsigned)((items + kThreads - 1) / kThreads)), dim3(kThreads),
-                   0, st, 1, ws, splits, M, N, C, ldc, out_bits, shift, (uint32_t)cpr);
+                   0, st, 1, ws, splits, M, N, C, ldc, out_bits, shift, cpr, rt);
 }
 
 }  // namespace gb300

@@ -73,7 +73,8 @@ namespace {
 // GB300_GEMM_BN (64, 96, 128, 192, 224 or 256; 64 and 96 for bf16 only)
 // forces the tile width,
 // GB300_GEMM_PAIR (0 or 1) the kernel family, GB300_GEMM_SPLITS (>= 1) the
-// split-K factor, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
+// split-K factor, GB300_GEMM_TAIL_SPLITS (0, or >= 2) the split tail of
+// the tensor-core kernels, GB300_GEMM_SKINNY_MAX_M the largest M sent to the
 // CUDA-core kernel, GB300_GEMM_TMA_STORE=0 direct stores (and scalar atomic
 // adds for the small-operand kernel's split-K), GB300_GEMM_PDL=0
 // plain stream ordering, GB300_GEMM_S8TM=0 the general int8 path for
@@ -84,6 +85,7 @@ struct Overrides {
   int bn = 0;            // 0: planner's choice
   int pair = -1;         // -1: planner's choice
   int splits = 0;        // 0: planner's choice
+  int tail_splits = -1;  // -1: planner's choice, 0: no split tail, >= 2: that split tail where one exists
   int skinny_max_m = -1; // -1: built-in limit
   bool tma_store = true;
   bool pdl = true;
@@ -102,6 +104,7 @@ Overrides read_overrides() {
   o.bn = env_int("GB300_GEMM_BN", 0);
   o.pair = env_int("GB300_GEMM_PAIR", -1);
   o.splits = env_int("GB300_GEMM_SPLITS", 0);
+  o.tail_splits = env_int("GB300_GEMM_TAIL_SPLITS", -1);
   o.skinny_max_m = env_int("GB300_GEMM_SKINNY_MAX_M", -1);
   o.tma_store = env_int("GB300_GEMM_TMA_STORE", 1) != 0;
   o.pdl = env_int("GB300_GEMM_PDL", 1) != 0;
@@ -371,13 +374,19 @@ struct Plan {
 // wins; on a tie the earlier candidate (single CTA before pair, wider before
 // narrower, fewer splits before more).  tile_model.choose_plan is the same
 // rule.
-double modelled_us(int64_t M, int64_t N, bool int8, bool pair, int bn, int64_t splits, int64_t kb_per,
-                   int64_t rounds) {
+//
+// A plan is costed by the work of its busiest CTA -- `steps` K steps in
+// `rounds` units -- and, when it writes split-K partials, the reduction
+// launch and the partials' bytes: tiles x splits units give rounds =
+// ceil(units / slots) of kb_per steps each; a split tail (the tiles of a
+// last, partly filled round split in tail_splits) gives the full rounds of
+// whole tiles plus one round of a tail unit's steps.
+double modelled_us(bool int8, bool pair, int bn, int64_t steps, int64_t rounds, double partial_mb) {
   const int wi = bn == 64 ? 0 : bn == 96 ? 1 : bn == 128 ? 2 : bn == 192 ? 3 : bn == 224 ? 4 : 5;
   const plan_table::StepCost c = plan_table::kCost[int8 ? 1 : 0][pair ? 1 : 0][wi];
-  double t = (double)rounds * ((double)kb_per * c.kstep_us + c.unit_us);
-  if (splits > 1)
-    t += plan_table::kSplitFixedUs[int8 ? 1 : 0] + plan_table::kSplitUsPerMB[int8 ? 1 : 0] * 4.0 * splits * M * N / 1e6;
+  double t = (double)steps * c.kstep_us + (double)rounds * c.unit_us;
+  if (partial_mb > 0)
+    t += plan_table::kSplitFixedUs[int8 ? 1 : 0] + plan_table::kSplitUsPerMB[int8 ? 1 : 0] * partial_mb;
   return t;
 }
 
@@ -396,7 +405,8 @@ double dram_us(int64_t M, int64_t N, int64_t K, bool int8, bool pair) {
   return (a_bytes + b_bytes * rb + c_bytes) / (plan_table::kHbmGBs * 1e3);
 }
 
-Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms, int pairs) {
+Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms, int pairs,
+               bool allow_tail = true) {
   Plan pl{};
   // compiled widths, widest first: the bf16 single-CTA kernels also come 64
   // and 96 wide (96 for B column-major only), for memory-bound GEMMs with
@@ -409,47 +419,72 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
   const int64_t num_kb = ceil_div(K, kBK);
   bool best_pair = false;
   int best_bn = 128;
-  int64_t best_splits = 1;
+  int64_t best_splits = 1, best_tail = 0, best_kb_tail = 0;
   double best_cost = -1.0, best_model = 0.0;
-  for (int fam = 0; fam < 2; ++fam) {
-    const bool pair = fam == 1;
-    if (pair && (M <= kBM || pairs <= 0)) continue;  // the second CTA would only compute padding
-    if (ovr.pair >= 0 && (ovr.pair != 0) != pair) continue;
-    const int *widths = b_kmajor ? kWidthsKMajor : (pair ? kPairWidthsMNMajor : kWidthsMNMajor);
-    const bool narrow = !pair && !int8;
-    const int nw = b_kmajor ? (narrow ? 6 : 4) : (pair ? 2 : (narrow ? 4 : 3));
-    const int64_t slots = pair ? pairs : sms;
-    const int64_t tiles_m = ceil_div(M, pair ? 2 * kBM : kBM);
-    for (int i = 0; i < nw; ++i) {
-      const int bn = widths[i];
-      if (N <= 128 && bn > 128) continue;
-      if (ovr.bn > 0 && ovr.bn != bn) continue;
-      const int64_t tiles = tiles_m * ceil_div(N, bn);
-      int64_t seen[17] = {};
-      int nseen = 0;
-      for (int64_t s = 1; s <= 16; ++s) {
-        int64_t kb_per = ceil_div(num_kb, s < num_kb ? s : num_kb);
-        int64_t s2 = ceil_div(num_kb, kb_per);
-        if (ovr.splits >= 1) {  // forced: exactly that split
-          if (s > 1) break;
-          const int64_t f = ovr.splits < num_kb ? ovr.splits : num_kb;
-          kb_per = ceil_div(num_kb, f);
-          s2 = ceil_div(num_kb, kb_per);
-        } else {
-          bool dup = false;
-          for (int j = 0; j < nseen; ++j) dup = dup || seen[j] == s2;
-          if (dup) continue;
-          if (s2 > 1 && (kb_per < 4 || tiles * s2 > 2 * slots)) continue;
+  const double mem_rank = plan_table::kMemWeight;
+  auto consider = [&](bool pair, int bn, int64_t splits, int64_t tail_splits, int64_t kb_tail, double model) {
+    const double cost = model + mem_rank * dram_us(M, N, K, int8, pair);
+    if (best_cost < 0 || cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best_model = model;
+      best_pair = pair;
+      best_bn = bn;
+      best_splits = splits;
+      best_tail = tail_splits;
+      best_kb_tail = kb_tail;
+    }
+  };
+  // A forced tail split (GB300_GEMM_TAIL_SPLITS >= 2) searches the split-tail
+  // plans alone first, and all plans only if none exists.
+  const bool tail_only_first = allow_tail && ovr.tail_splits >= 2;
+  for (int pass = tail_only_first ? 0 : 1; pass < 2 && best_cost < 0; ++pass) {
+    const bool tail_only = pass == 0;
+    for (int fam = 0; fam < 2; ++fam) {
+      const bool pair = fam == 1;
+      if (pair && (M <= kBM || pairs <= 0)) continue;  // the second CTA would only compute padding
+      if (ovr.pair >= 0 && (ovr.pair != 0) != pair) continue;
+      const int *widths = b_kmajor ? kWidthsKMajor : (pair ? kPairWidthsMNMajor : kWidthsMNMajor);
+      const bool narrow = !pair && !int8;
+      const int nw = b_kmajor ? (narrow ? 6 : 4) : (pair ? 2 : (narrow ? 4 : 3));
+      const int64_t slots = pair ? pairs : sms;
+      const int64_t tiles_m = ceil_div(M, pair ? 2 * kBM : kBM);
+      for (int i = 0; i < nw; ++i) {
+        const int bn = widths[i];
+        if (N <= 128 && bn > 128) continue;
+        if (ovr.bn > 0 && ovr.bn != bn) continue;
+        const int64_t tiles = tiles_m * ceil_div(N, bn);
+        int64_t seen[17] = {};
+        int nseen = 0;
+        for (int64_t s = 1; s <= 16 && !tail_only; ++s) {
+          int64_t kb_per = ceil_div(num_kb, s < num_kb ? s : num_kb);
+          int64_t s2 = ceil_div(num_kb, kb_per);
+          if (ovr.splits >= 1) {  // forced: exactly that split
+            if (s > 1) break;
+            const int64_t f = ovr.splits < num_kb ? ovr.splits : num_kb;
+            kb_per = ceil_div(num_kb, f);
+            s2 = ceil_div(num_kb, kb_per);
+          } else {
+            bool dup = false;
+            for (int j = 0; j < nseen; ++j) dup = dup || seen[j] == s2;
+            if (dup) continue;
+            if (s2 > 1 && (kb_per < 4 || tiles * s2 > 2 * slots)) continue;
+          }
+          seen[nseen++] = s2;
+          const int64_t rounds = ceil_div(tiles * s2, slots);
+          consider(pair, bn, s2, 0, 0,
+                   modelled_us(int8, pair, bn, rounds * kb_per, rounds, s2 > 1 ? 4.0 * s2 * M * N / 1e6 : 0.0));
         }
-        seen[nseen++] = s2;
-        const double model = modelled_us(M, N, int8, pair, bn, s2, kb_per, ceil_div(tiles * s2, slots));
-        const double cost = model + plan_table::kMemWeight * dram_us(M, N, K, int8, pair);
-        if (best_cost < 0 || cost < best_cost - 1e-9) {
-          best_cost = cost;
-          best_model = model;
-          best_pair = pair;
-          best_bn = bn;
-          best_splits = s2;
+        // Split tail: whole tiles for the full rounds, the last round's
+        // tiles (at most half a round of them) split in S so that they fill
+        // it; S = 2 .. 8 with at least 4 K steps a unit.
+        const int64_t full = tiles / slots, tail = tiles - full * slots;
+        if (!allow_tail || ovr.tail_splits == 0 || ovr.splits > 1 || full < 1 || tail == 0) continue;
+        for (int64_t st2 = 2; st2 <= 8 && tail * st2 <= slots; ++st2) {
+          if (ovr.tail_splits >= 2 && st2 != ovr.tail_splits) continue;
+          const int64_t kb_tail = ceil_div(num_kb, st2);
+          if (ceil_div(num_kb, kb_tail) != st2 || kb_tail < 4) continue;
+          const double part_mb = 4.0 * st2 * tail * (pair ? 2 * kBM : kBM) * bn / 1e6;
+          consider(pair, bn, 1, st2, kb_tail, modelled_us(int8, pair, bn, full * num_kb + kb_tail, full + 1, part_mb));
         }
       }
     }
@@ -462,6 +497,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
   const int64_t tiles = tiles_m * tiles_n;
   const int64_t kb_per = ceil_div(num_kb, best_splits);
   const int64_t splits = ceil_div(num_kb, kb_per);
+  const int64_t full_rounds = best_tail > 0 ? tiles / slots : 0;
   // Output path: the bf16 224-wide kernels keep a pipeline stage and stage
   // their TMA stores through 1 KB blocks; for int8 at 192/224, TMA stores
   // (4 KB blocks, one stage less) win up to 128 K steps per unit, beyond
@@ -488,23 +524,33 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, bool b_kmajor, int epi, int sms,
   p.group_m = 8;
   p.out_bits = 32;
   p.out_shift = 0;
-  const int64_t units = tiles * splits;
+  p.tail_first = (int)(full_rounds * slots);
+  p.tail_splits = (int)best_tail;
+  p.tail_kb_per = (int)best_kb_tail;
+  p.ws_tma = 0;
+  const int64_t units = best_tail > 0 ? full_rounds * slots + (tiles - full_rounds * slots) * best_tail
+                                      : tiles * splits;
   const int64_t used = units < slots ? units : slots;
   pl.grid = (int)(pair ? 2 * used : used);
   if (ovr.debug)
     std::fprintf(stderr,
-                 "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d%s tiles=%lldx%lld splits=%lld grid=%d "
-                 "model %.1f us (SMs %d, co-resident pairs %d)\n",
+                 "[gb300_gemm] M=%lld N=%lld K=%lld %s B%s: %s BN=%d%s tiles=%lldx%lld splits=%lld "
+                 "tail splits=%lld from tile %d grid=%d model %.1f us (SMs %d, co-resident pairs %d)\n",
                  (long long)M, (long long)N, (long long)K, epi == kEpiS32 ? "int8" : "bf16",
                  b_kmajor ? "col" : "row", pair ? "pair" : "single", bn,
                  tma_out == 2 ? " tma-store-1k" : tma_out ? " tma-store" : "", (long long)tiles_m,
-                 (long long)tiles_n, (long long)splits, pl.grid, best_model, sms, pairs);
+                 (long long)tiles_n, (long long)splits, (long long)best_tail, p.tail_first, pl.grid, best_model, sms,
+                 pairs);
   return pl;
 }
 
 struct WsLayout {
   size_t a_off = 0, b_off = 0, part_off = 0, total = 0;
 };
+
+// Planes of M x N 32-bit partials a plan writes (split-K, or a split tail,
+// which writes only its tiles' parts of them); 0 when C is written directly.
+int64_t partial_planes(const TcParams &p) { return p.splits > 1 ? p.splits : p.tail_splits; }
 
 // Shared path after staging: encode maps, launch the tcgen05 kernel and the
 // split-K reduction.
@@ -539,8 +585,16 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   // An output that will be stored directly wants the variant with the extra
   // pipeline stage where one exists (int8 at 192 / 224).
   if (!tma_ok && s32 && (pl.v.bn == 192 || pl.v.bn == 224)) pl.v.tma_out = 0;
-  CUtensorMap tout = tb;
+  CUtensorMap tout = tb, tws = tb;
   p.out_tma = kOutDirect;
+  p.ws_tma = 0;
+  // a split tail's partials go through TMA where split-K partials would
+  if (p.tail_splits > 0 && pl.v.tma_out == 1 && p.N % 4 == 0 && overrides().tma_store) {
+    if (!encode_out(&tws, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, partials,
+                    (uint64_t)p.N, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.tail_splits))
+      return cuda_failed("tail partials tensor map");
+    p.ws_tma = 1;
+  }
   if (pl.v.tma_out != 0 && tma_ok) {
     if (p.splits > 1) {
       if (p.N % 4 == 0) {
@@ -566,20 +620,26 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   if (prof && cudaEventRecord(g_prof_start, st) != cudaSuccess) return GEMM_ERR_CUDA;
   cudaError_t e;
   if (pl.v.pair)
-    e = pl.v.epi == kEpiS32 ? launch_tc2_s32(pl.v, ta, tb, tout, p, pl.grid, st)
-                            : launch_tc2_bf16(pl.v, ta, tb, tout, p, pl.grid, st);
+    e = pl.v.epi == kEpiS32 ? launch_tc2_s32(pl.v, ta, tb, tout, tws, p, pl.grid, st)
+                            : launch_tc2_bf16(pl.v, ta, tb, tout, tws, p, pl.grid, st);
   else
-    e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, tout, p, pl.grid, st)
-                            : launch_tc_bf16(pl.v, ta, tb, tout, p, pl.grid, st);
+    e = pl.v.epi == kEpiS32 ? launch_tc_s32(pl.v, ta, tb, tout, tws, p, pl.grid, st)
+                            : launch_tc_bf16(pl.v, ta, tb, tout, tws, p, pl.grid, st);
   g_launches.fetch_add(1);
   if (e != cudaSuccess) return cuda_failed(pl.v.pair ? "CTA-pair kernel launch" : "tensor-core kernel launch", e);
   if (prof && cudaEventRecord(g_prof_stop, st) != cudaSuccess) return GEMM_ERR_CUDA;
-  if (p.splits > 1) {
+  const int planes = (int)partial_planes(p);
+  if (planes > 0) {
+    ReduceTiles rt{0, 0, p.tiles_m, p.tiles_n, p.group_m, pl.v.pair ? 2 * kBM : kBM, pl.v.bn};
+    if (p.tail_splits > 0) {  // only the split tail's tiles
+      rt.first = p.tail_first;
+      rt.count = p.tiles_m * p.tiles_n - p.tail_first;
+    }
     e = pl.v.epi == kEpiS32
-            ? launch_splitk_reduce_s32(static_cast<const int32_t *>(partials), p.splits, p.M, p.N, C, ldc,
-                                       p.out_bits, p.out_shift, d.sms, st)
-            : launch_splitk_reduce_bf16(static_cast<const float *>(partials), p.splits, p.M, p.N,
-                                        static_cast<uint16_t *>(C), ldc, d.sms, st);
+            ? launch_splitk_reduce_s32(static_cast<const int32_t *>(partials), planes, p.M, p.N, C, ldc,
+                                       p.out_bits, p.out_shift, rt, st)
+            : launch_splitk_reduce_bf16(static_cast<const float *>(partials), planes, p.M, p.N,
+                                        static_cast<uint16_t *>(C), ldc, rt, st);
     g_launches.fetch_add(1);
     if (e != cudaSuccess) return GEMM_ERR_CUDA;
   }
@@ -594,7 +654,7 @@ constexpr int64_t kTinyMaxMacs = int64_t(1) << 27;  // 512^3
 int64_t tiny_max_macs() {
   const Overrides o = overrides();
   // a forced tile width, family or split asks for the tensor-core kernels
-  if (o.bn > 0 || o.pair >= 0 || o.splits >= 1) return 0;
+  if (o.bn > 0 || o.pair >= 0 || o.splits >= 1 || o.tail_splits >= 2) return 0;
   return o.tiny_max_macs >= 0 ? o.tiny_max_macs : kTinyMaxMacs;
 }
 
@@ -676,7 +736,10 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
   size_t off = 0;
   if (pack_a) { L.a_off = off; off = align_up(off + (size_t)M * lda_p * 2, 256); }
   if (pack_b) { L.b_off = off; off = align_up(off + (size_t)b_rows * ldb_p * 2, 256); }
-  if (pl.p.splits > 1) { L.part_off = off; off = align_up(off + (size_t)pl.p.splits * M * N * 4, 256); }
+  if (partial_planes(pl.p) > 0) {
+    L.part_off = off;
+    off = align_up(off + (size_t)partial_planes(pl.p) * M * N * 4, 256);
+  }
   L.total = off;
   if (L.total && (s = ensure_workspace(L.total, st)) != GEMM_OK) return s;
   uint8_t *ws = static_cast<uint8_t *>(scratch_ws());
@@ -696,7 +759,8 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
     Bu = dst;
     ldb_u = ldb_p;
   }
-  return run_tc(*d, pl, Au, lda_u, Bu, ldb_u, C, ldc, 2, pl.p.splits > 1 ? ws + L.part_off : nullptr, st);
+  return run_tc(*d, pl, Au, lda_u, Bu, ldb_u, C, ldc, 2, partial_planes(pl.p) > 0 ? ws + L.part_off : nullptr,
+                st);
 }
 
 }  // extern "C"
@@ -869,7 +933,7 @@ bool try_s8tm(DeviceState &d, int64_t M, int64_t N, int64_t K, const int8_t *A, 
   if (splits > 1 && !add_into_c) {
     g_launches.fetch_add(1);
     if (launch_splitk_reduce_s32(static_cast<const int32_t *>(p.ws), (int)splits, M, N, C, ldc, out_bits, shift,
-                                 d.sms, st) != cudaSuccess)
+                                 ReduceTiles{}, st) != cudaSuccess)
       return true;
   }
   *status = GEMM_OK;
@@ -921,7 +985,10 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   off = align_up(off + (size_t)M * lda_p * 2, 256);
   L.b_off = off;
   off = align_up(off + (size_t)b_rows * ldb_p * 2, 256);
-  if (pl.p.splits > 1) { L.part_off = off; off = align_up(off + (size_t)pl.p.splits * M * N * 4, 256); }
+  if (partial_planes(pl.p) > 0) {
+    L.part_off = off;
+    off = align_up(off + (size_t)partial_planes(pl.p) * M * N * 4, 256);
+  }
   L.total = off;
   if ((s = ensure_workspace(L.total, st)) != GEMM_OK) return s;
   uint8_t *ws = static_cast<uint8_t *>(scratch_ws());
@@ -931,8 +998,8 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   if (launch_s8_to_bf16_pair(S8Job{A, M, K, lda, Ab, lda_p}, S8Job{B, b_rows, b_cols, ldb, Bb, ldb_p}, d->sms,
                              st) != cudaSuccess)
     return GEMM_ERR_CUDA;
-  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, out_esize, pl.p.splits > 1 ? ws + L.part_off : nullptr,
-                st);
+  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, out_esize,
+                partial_planes(pl.p) > 0 ? ws + L.part_off : nullptr, st);
 }
 
 }  // namespace
@@ -1063,6 +1130,7 @@ gemm_status_t gemm_plan_query(int64_t M, int64_t N, int64_t K, int int8, int b_l
   out->route = pl.v.pair ? GEMM_ROUTE_TC_PAIR : GEMM_ROUTE_TC_SINGLE;
   out->bn = pl.v.bn;
   out->splits = pl.p.splits;
+  out->tail_splits = pl.p.tail_splits;
   out->stages = tc_max_stages(pl.v.pair ? pl.v.bn / 2 : pl.v.bn, ew, pl.v.tma_out);
   out->grid = pl.grid;
   out->model_us = pl.model_us;
@@ -1122,7 +1190,15 @@ gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t
   const size_t a_off = 0;
   const size_t b_off = align_up((size_t)M * lda_p * 2, 256);
   const size_t part_off = align_up(b_off + (size_t)b_rows * ldb_p * 2, 256);
-  const size_t total = pl.p.splits > 1 ? align_up(part_off + (size_t)pl.p.splits * M * N * 4, 256) : part_off;
+  auto total_of = [&](const Plan &q) {
+    const int64_t planes = partial_planes(q.p);
+    return planes > 0 ? align_up(part_off + (size_t)planes * M * N * 4, 256) : part_off;
+  };
+  // a split tail's partial planes may not fit the caller's scratch: plan
+  // without one then
+  if (pl.p.tail_splits > 0 && total_of(pl) > capacity)
+    pl = make_plan(M, N, K, b_kmajor, kEpiS32, d->sms, pair_slots(), false);
+  const size_t total = total_of(pl);
   if (!scratch || total > capacity) return GEMM_ERR_UNSUPPORTED;
   uint8_t *ws = static_cast<uint8_t *>(scratch);
   uint16_t *Ab = reinterpret_cast<uint16_t *>(ws + a_off);
@@ -1131,7 +1207,7 @@ gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t
   if (launch_s8_to_bf16_pair(S8Job{A, M, K, lda, Ab, lda_p}, S8Job{B, b_rows, b_cols, ldb, Bb, ldb_p}, d->sms,
                              st) != cudaSuccess)
     return GEMM_ERR_CUDA;
-  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, pl.p.splits > 1 ? ws + part_off : nullptr, st);
+  return run_tc(*d, pl, Ab, lda_p, Bb, ldb_p, C, ldc, 4, partial_planes(pl.p) > 0 ? ws + part_off : nullptr, st);
 }
 
 }  // namespace gb300

@@ -58,9 +58,9 @@ struct TcVariant {
 
 // Launch the persistent tcgen05 GEMM kernel (gemm_tc_bf16.cu / gemm_tc_s32.cu).
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
+                           const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st);
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                          const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
+                          const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st);
 // Output variant (TcVariant::tma_out) of the bf16 kernel of a tile width.
 int tc_bf16_tma_out(int bn);
 int tc2_bf16_tma_out(int bn);
@@ -68,9 +68,9 @@ int tc2_bf16_tma_out(int bn);
 int pair_slots();
 // The CTA-pair kernel (gemm_tc2_bf16.cu / gemm_tc2_s32.cu); grid is even.
 cudaError_t launch_tc2_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
+                            const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st);
 cudaError_t launch_tc2_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st);
+                           const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st);
 
 // int8 GEMM for memory-bound shapes with the large operand converted to bf16
 // inside the kernel (gemm_s8tm.cu).  P (int8, K contiguous, P_rows x K) is
@@ -138,13 +138,21 @@ cudaError_t launch_wait_timeout_probe(uint32_t *err, uint64_t limit_ns, cudaStre
 // Fill an M x N block of 8-, 16- or 32-bit elements with zero.
 cudaError_t launch_zero_fill(void *C, int64_t M, int64_t N, int64_t ldc, int esize, int sms,
                              cudaStream_t st);
+// The part of C a split-K reduction covers: all of it (count == 0), or the
+// `count` tiles of rows x cols (cols a multiple of 4) from raster position
+// `first` on (raster_tile), the split tail of a tensor-core launch.
+struct ReduceTiles {
+  int first, count, tiles_m, tiles_n, group_m, rows, cols;
+};
 // Split-K reduction: C = round(sum over splits of ws[s]) (fp32 -> bf16 RNE)
 // or C = sum of int32 partials, stored as int32 (out_bits 32) or
-// requantised to out_bits = 16 / 8 with right shift `shift`.
+// requantised to out_bits = 16 / 8 with right shift `shift`; over the
+// elements of C that rt covers.
 cudaError_t launch_splitk_reduce_bf16(const float *ws, int splits, int64_t M, int64_t N,
-                                      uint16_t *C, int64_t ldc, int sms, cudaStream_t st);
+                                      uint16_t *C, int64_t ldc, const ReduceTiles &rt, cudaStream_t st);
 cudaError_t launch_splitk_reduce_s32(const int32_t *ws, int splits, int64_t M, int64_t N, void *C,
-                                     int64_t ldc, int out_bits, int shift, int sms, cudaStream_t st);
+                                     int64_t ldc, int out_bits, int shift, const ReduceTiles &rt,
+                                     cudaStream_t st);
 
 // Argument checks of the int8 entry points (no CUDA calls).
 gemm_status_t validate_s8(int64_t M, int64_t N, int64_t K, const void *A, int64_t lda, const void *B,

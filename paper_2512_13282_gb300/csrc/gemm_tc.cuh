@@ -71,6 +71,14 @@ struct TcParams {
   int out_bits;      // int8 path: 32 (exact int32 C), 16 or 8 (requantised C)
   int out_shift;     // int8 path with out_bits < 32: right shift, 0..31
   int out_tma;       // kOutDirect, kOutTmaC (tmOut maps C) or kOutTmaWs (tmOut maps the partials)
+  // Split tail (tail_splits >= 2, splits == 1): the tiles of the last,
+  // partly filled round -- raster positions tail_first .. -- are each split
+  // into tail_splits units of tail_kb_per k-blocks that write partials
+  // (planes as for split-K) for the reduction kernel, so that the round
+  // takes 1 / tail_splits of a tile's time; every other tile is one unit
+  // writing C.  tail_first is a whole number of rounds of units.  ws_tma:
+  // the partials are stored through tmWs (else directly).
+  int tail_first, tail_splits, tail_kb_per, ws_tma;
 };
 
 // How the epilogue writes its results.
@@ -130,25 +138,54 @@ struct TcCfg {
 
 struct Unit {
   int tm, tn, split, kb0, kb1;
+  int part;  // 1: the unit writes split-K partials (plane `split`), 0: C
 };
 
-// Work unit u -> (tile, split).  Tiles are visited in groups of group_m
-// M-tiles so that CTAs running at the same time share A rows and B columns
-// in L2.
+// Raster position t -> output tile (tm, tn).  Tiles are visited in groups of
+// group_m M-tiles so that CTAs running at the same time share A rows and B
+// columns in L2.  The split-K reduction of a split tail walks the same
+// positions.
+__host__ __device__ __forceinline__ void raster_tile(int t, int tiles_m, int tiles_n, int group_m, int *tm,
+                                                     int *tn) {
+  const int group = group_m * tiles_n;
+  const int gid = t / group;
+  const int first_m = gid * group_m;
+  const int gm = tiles_m - first_m < group_m ? tiles_m - first_m : group_m;
+  const int local = t - gid * group;
+  *tm = first_m + local % gm;
+  *tn = local / gm;
+}
+
+// Work units of a launch: tiles x splits, or the whole tiles before the
+// split tail plus tail_splits units per tail tile.
+__device__ __forceinline__ int tc_num_units(const TcParams &p) {
+  const int num_tiles = p.tiles_m * p.tiles_n;
+  return p.tail_splits > 0 ? p.tail_first + (num_tiles - p.tail_first) * p.tail_splits : num_tiles * p.splits;
+}
+
+// Work unit u -> (tile, split, k-blocks).  With split-K, unit u is split
+// u / tiles of raster position u % tiles; with a split tail, units below
+// tail_first are whole tiles and the rest split the tail tiles.
 __device__ __forceinline__ Unit decode_unit(const TcParams &p, int u) {
   const int num_tiles = p.tiles_m * p.tiles_n;
   Unit w;
-  w.split = u / num_tiles;
-  const int t = u - w.split * num_tiles;
-  const int group = p.group_m * p.tiles_n;
-  const int gid = t / group;
-  const int first_m = gid * p.group_m;
-  const int gm = min(p.tiles_m - first_m, p.group_m);
-  const int local = t - gid * group;
-  w.tm = first_m + local % gm;
-  w.tn = local / gm;
-  w.kb0 = w.split * p.kb_per_split;
-  w.kb1 = min(p.num_kb, w.kb0 + p.kb_per_split);
+  int t;
+  if (p.tail_splits > 0 && u >= p.tail_first) {
+    const int tail = num_tiles - p.tail_first;
+    const int v = u - p.tail_first;
+    w.split = v / tail;
+    t = p.tail_first + (v - w.split * tail);
+    w.kb0 = w.split * p.tail_kb_per;
+    w.kb1 = min(p.num_kb, w.kb0 + p.tail_kb_per);
+    w.part = 1;
+  } else {
+    w.split = u / num_tiles;
+    t = u - w.split * num_tiles;
+    w.kb0 = w.split * p.kb_per_split;
+    w.kb1 = min(p.num_kb, w.kb0 + p.kb_per_split);
+    w.part = p.splits > 1 ? 1 : 0;
+  }
+  raster_tile(t, p.tiles_m, p.tiles_n, p.group_m, &w.tm, &w.tn);
   return w;
 }
 
@@ -425,9 +462,12 @@ __device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[W]) {
 template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmOut, const TcParams p) {
+                   const __grid_constant__ CUtensorMap tmOut, const __grid_constant__ CUtensorMap tmWs,
+                   const TcParams p) {
   using Cfg = TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>;
   const int out_tma = TMA_OUT != 0 ? p.out_tma : (int)kOutDirect;
+  // the split tail's partials: through tmWs by the 4 KB staging blocks, or directly
+  const int tail_out = (TMA_OUT == 1 && p.ws_tma) ? (int)kOutTmaWs : (int)kOutDirect;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // swizzle atoms need 1024-byte alignment
@@ -462,6 +502,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
     if (out_tma != kOutDirect) tma_prefetch_desc(&tmOut);
+    if (p.tail_splits > 0 && tail_out != kOutDirect) tma_prefetch_desc(&tmWs);
   }
   if (warp == 1) tmem_alloc<Cfg::kTmemCols>(smem_addr(tmem_slot));
   tc_fence_before_sync();
@@ -473,7 +514,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
   // global memory is touched only after that kernel has completed.
   griddep_wait();
 
-  const int num_units = p.tiles_m * p.tiles_n * p.splits;
+  const int num_units = tc_num_units(p);
   constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
 
   if (warp == 0) {
@@ -564,13 +605,16 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
     const int quad = warp & 3;  // a warp may only touch TMEM lanes 32*(warp%4) ..
     const int colpart = ew >> 2;
     const int row_in_tile = quad * 32 + lane;
-    const bool split = p.splits > 1;
     const bool ws_vec = (p.N & 3) == 0;
     const uint32_t ebuf = base + Cfg::kEpiOffset + ew * Cfg::kEpiWarpBytes;
     uint32_t acc_cnt = 0;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < num_units; u += gridDim.x) {
       const Unit w = decode_unit(p, u);
+      const bool split = w.part != 0;                  // partials of this unit, not C
+      const bool tail = split && p.tail_splits > 0;    // ... of a split-tail tile
+      const int uo = tail ? tail_out : out_tma;
+      const CUtensorMap *om = tail ? &tmWs : &tmOut;
       const int64_t row = (int64_t)w.tm * kBM + row_in_tile;
       const bool row_ok = row < p.M;
       const int col0 = w.tn * BN + colpart * CPT;
@@ -596,7 +640,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
             tmem_ld_wait();
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(__float2int_rn(__uint_as_float(v[i])));
-            store_s32_chunk(p, &tmOut, ebuf, lane, out_tma, v, col0 + c * 32, y0, w.split, row_ok, row, wrow, ws_vec);
+            store_s32_chunk(p, om, ebuf, lane, uo, v, col0 + c * 32, y0, w.split, row_ok, row, wrow, ws_vec);
           }
           if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
             constexpr int kTail = (CPT / 32) * 32;
@@ -653,19 +697,19 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
         // split-K partials stay int32; the reduction requantises
         uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
                                : nullptr;
-        if (out_tma != kOutDirect) {
+        if (uo != kOutDirect) {
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
             const int x = col0 + c * 32;
-            if (out_tma == kOutTmaWs)
-              tma_out_words32<true>(&tmOut, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
+            if (uo == kOutTmaWs)
+              tma_out_words32<true>(om, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
             else if (p.out_bits == 32)
-              tma_out_words32<false>(&tmOut, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+              tma_out_words32<false>(om, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
             else
-              tma_out_narrow(&tmOut, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
+              tma_out_narrow(om, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
           }
           if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
             constexpr int kTail = (CPT / 32) * 32;
@@ -718,12 +762,12 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
           tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
           const int x = col0 + c * 32;
-          if (TMA_OUT == 1 && out_tma == kOutTmaWs) {
-            tma_out_words32<true>(&tmOut, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
-          } else if (TMA_OUT == 1 && out_tma == kOutTmaC) {
-            tma_out_bf16x32(&tmOut, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
-          } else if (TMA_OUT == 2 && out_tma == kOutTmaC) {
-            tma_out_bf16x16x2(&tmOut, ebuf, lane, r, x, y0, p.M, p.N);
+          if (TMA_OUT == 1 && uo == kOutTmaWs) {
+            tma_out_words32<true>(om, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
+          } else if (TMA_OUT == 1 && uo == kOutTmaC) {
+            tma_out_bf16x32(om, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
+          } else if (TMA_OUT == 2 && uo == kOutTmaC) {
+            tma_out_bf16x16x2(om, ebuf, lane, r, x, y0, p.M, p.N);
           } else if (row_ok) {
             if (split)
               store_words<32>(wrow, x, p.N, ws_vec, r);

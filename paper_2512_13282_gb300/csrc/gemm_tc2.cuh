@@ -118,9 +118,12 @@ struct Tc2Cfg {
 template <int BN, int STAGES, bool B_KMAJOR, int EPI, int EPI_WARPS, int TMA_OUT>
 __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>::kThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const __grid_constant__ CUtensorMap tmOut, const TcParams p) {
+                    const __grid_constant__ CUtensorMap tmOut, const __grid_constant__ CUtensorMap tmWs,
+                    const TcParams p) {
   using Cfg = Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TMA_OUT>;
   const int out_tma = TMA_OUT != 0 ? p.out_tma : (int)kOutDirect;
+  // the split tail's partials: through tmWs by the 4 KB staging blocks, or directly
+  const int tail_out = (TMA_OUT == 1 && p.ws_tma) ? (int)kOutTmaWs : (int)kOutDirect;
   constexpr int kTileM = 2 * kBM;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -160,6 +163,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
     if (out_tma != kOutDirect) tma_prefetch_desc(&tmOut);
+    if (p.tail_splits > 0 && tail_out != kOutDirect) tma_prefetch_desc(&tmWs);
   }
   __syncwarp();
   if (warp == 1) tmem_alloc_pair<Cfg::kTmemCols>(smem_addr(tmem_slot));
@@ -172,7 +176,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
   // global memory is touched only after that kernel has completed.
   griddep_wait();
 
-  const int num_units = p.tiles_m * p.tiles_n * p.splits;
+  const int num_units = tc_num_units(p);
   constexpr uint64_t kDrainNs = 200ull * 1000 * 1000;
 
   if (warp == 0) {
@@ -268,13 +272,16 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
     const int quad = warp & 3;
     const int colpart = ew >> 2;
     const int row_in_tile = (int)rank * kBM + quad * 32 + lane;
-    const bool split = p.splits > 1;
     const bool ws_vec = (p.N & 3) == 0;
     const uint32_t ebuf = base + Cfg::kEpiOffset + ew * Cfg::kEpiWarpBytes;
     uint32_t acc_cnt = 0;
     bool ok = true;
     for (int u = cluster; ok && u < num_units; u += num_clusters) {
       const Unit w = decode_unit(p, u);
+      const bool split = w.part != 0;                  // partials of this unit, not C
+      const bool tail = split && p.tail_splits > 0;    // ... of a split-tail tile
+      const int uo = tail ? tail_out : out_tma;
+      const CUtensorMap *om = tail ? &tmWs : &tmOut;
       const int64_t row = (int64_t)w.tm * kTileM + row_in_tile;
       const bool row_ok = row < p.M;
       const int col0 = w.tn * BN + colpart * CPT;
@@ -315,19 +322,19 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
         // split-K partials stay int32; the reduction requantises
         uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
                                : nullptr;
-        if (out_tma != kOutDirect) {
+        if (uo != kOutDirect) {
 #pragma unroll
           for (int c = 0; c < CPT / 32; ++c) {
             uint32_t v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
             const int x = col0 + c * 32;
-            if (out_tma == kOutTmaWs)
-              tma_out_words32<true>(&tmOut, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
+            if (uo == kOutTmaWs)
+              tma_out_words32<true>(om, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
             else if (p.out_bits == 32)
-              tma_out_words32<false>(&tmOut, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
+              tma_out_words32<false>(om, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
             else
-              tma_out_narrow(&tmOut, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
+              tma_out_narrow(om, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
           }
           if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
             constexpr int kTail = (CPT / 32) * 32;
@@ -380,12 +387,12 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
           tmem_ld<32>(t0 + c * 32, r);
           tmem_ld_wait();
           const int x = col0 + c * 32;
-          if (TMA_OUT == 1 && out_tma == kOutTmaWs) {
-            tma_out_words32<true>(&tmOut, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
-          } else if (TMA_OUT == 1 && out_tma == kOutTmaC) {
-            tma_out_bf16x32(&tmOut, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
-          } else if (TMA_OUT == 2 && out_tma == kOutTmaC) {
-            tma_out_bf16x16x2(&tmOut, ebuf, lane, r, x, y0, p.M, p.N);
+          if (TMA_OUT == 1 && uo == kOutTmaWs) {
+            tma_out_words32<true>(om, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
+          } else if (TMA_OUT == 1 && uo == kOutTmaC) {
+            tma_out_bf16x32(om, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
+          } else if (TMA_OUT == 2 && uo == kOutTmaC) {
+            tma_out_bf16x16x2(om, ebuf, lane, r, x, y0, p.M, p.N);
           } else if (row_ok) {
             if (split)
               store_words<32>(wrow, x, p.N, ws_vec, r);

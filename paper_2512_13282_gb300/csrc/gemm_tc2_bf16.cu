@@ -8,18 +8,18 @@ namespace gb300 {
 // 4 KB staging blocks, or 1 KB blocks for 224, which keeps its seventh stage.
 // Every kernel takes the deepest ring that fits (tc_max_stages: 6, 7, 7, 8).
 cudaError_t launch_tc2_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                            const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
+                            const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_pair<256, tc_max_stages(256 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 224: return launch_pair<224, tc_max_stages(224 / 2, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
-      case 192: return launch_pair<192, tc_max_stages(192 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_pair<128, tc_max_stages(128 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_pair<256, tc_max_stages(256 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 224: return launch_pair<224, tc_max_stages(224 / 2, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, w, p, grid, st);
+      case 192: return launch_pair<192, tc_max_stages(192 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 128: return launch_pair<128, tc_max_stages(128 / 2, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_pair<256, tc_max_stages(256 / 2, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_pair<128, tc_max_stages(128 / 2, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_pair<256, tc_max_stages(256 / 2, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 128: return launch_pair<128, tc_max_stages(128 / 2, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;

@@ -7,7 +7,7 @@
 namespace gb300 {
 
 template <int BN, int STAGES, bool KM, int EPI, int EW, int TMA>
-cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
+cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const CUtensorMap &w, const TcParams &p,
                         int grid,
                         cudaStream_t st) {
   using Cfg = Tc2Cfg<BN, STAGES, KM, EPI, EW, TMA>;
@@ -22,7 +22,7 @@ cudaError_t launch_pair(const CUtensorMap &a, const CUtensorMap &b, const CUtens
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
   // grid is even: a whole number of pairs
-  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 2, a, b, o, p);
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 2, a, b, o, w, p);
 }
 
 }  // namespace gb300

@@ -5,7 +5,7 @@ namespace gb300 {
 
 namespace {
 template <int BN, int STAGES, bool KM, int EPI, int EW, int TMA>
-cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
+cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const CUtensorMap &w, const TcParams &p,
                        int grid,
                        cudaStream_t st) {
   using Cfg = TcCfg<BN, STAGES, KM, EPI, EW, TMA>;
@@ -20,7 +20,7 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
-  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, o, p);
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, o, w, p);
 }
 }  // namespace
 
@@ -34,22 +34,22 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 // without a K split, and so without the reduction launch (bf16 128 x 11008
 // x 4096: 115 CTAs), and 64 fits N = 64 without padding columns.
 cudaError_t launch_tc_bf16(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                           const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
+                           const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st) {
   if (v.b_kmajor) {
     switch (v.bn) {
-      case 256: return launch_one<256, tc_max_stages(256, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 224: return launch_one<224, tc_max_stages(224, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, p, grid, st);
-      case 192: return launch_one<192, tc_max_stages(192, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_one<128, tc_max_stages(128, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 96: return launch_one<96, tc_max_stages(96, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 64: return launch_one<64, tc_max_stages(64, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_one<256, tc_max_stages(256, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 224: return launch_one<224, tc_max_stages(224, 4, 2), true, kEpiBf16, 4, 2>(a, b, o, w, p, grid, st);
+      case 192: return launch_one<192, tc_max_stages(192, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 128: return launch_one<128, tc_max_stages(128, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 96: return launch_one<96, tc_max_stages(96, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 64: return launch_one<64, tc_max_stages(64, 4, 1), true, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
     }
   } else {
     switch (v.bn) {
-      case 256: return launch_one<256, tc_max_stages(256, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 192: return launch_one<192, tc_max_stages(192, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 128: return launch_one<128, tc_max_stages(128, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
-      case 64: return launch_one<64, tc_max_stages(64, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, p, grid, st);
+      case 256: return launch_one<256, tc_max_stages(256, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 192: return launch_one<192, tc_max_stages(192, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 128: return launch_one<128, tc_max_stages(128, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
+      case 64: return launch_one<64, tc_max_stages(64, 4, 1), false, kEpiBf16, 4, 1>(a, b, o, w, p, grid, st);
     }
   }
   return cudaErrorInvalidValue;

@@ -5,7 +5,7 @@ namespace gb300 {
 
 namespace {
 template <int BN, int STAGES, bool KM, int EPI, int EW, int TMA>
-cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const TcParams &p,
+cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtensorMap &o, const CUtensorMap &w, const TcParams &p,
                        int grid,
                        cudaStream_t st) {
   using Cfg = TcCfg<BN, STAGES, KM, EPI, EW, TMA>;
@@ -20,7 +20,7 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) opted_in[dev] = true;
   }
-  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, o, p);
+  return launch_ex(kern, dim3((unsigned)grid), dim3(Cfg::kThreads), Cfg::kSmemBytes, st, 1, a, b, o, w, p);
 }
 }  // namespace
 
@@ -32,23 +32,23 @@ cudaError_t launch_one(const CUtensorMap &a, const CUtensorMap &b, const CUtenso
 // long reductions prefer (the planner's choice, v.tma_out).  Every kernel
 // takes the deepest ring that fits (tc_max_stages).
 cudaError_t launch_tc_s32(const TcVariant &v, const CUtensorMap &a, const CUtensorMap &b,
-                          const CUtensorMap &o, const TcParams &p, int grid, cudaStream_t st) {
+                          const CUtensorMap &o, const CUtensorMap &w, const TcParams &p, int grid, cudaStream_t st) {
   const bool km = v.b_kmajor, t = v.tma_out != 0;
   switch (v.bn) {
-    case 256: return km ? launch_one<256, tc_max_stages(256, 8, 1), true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-                        : launch_one<256, tc_max_stages(256, 8, 1), false, kEpiS32, 8, 1>(a, b, o, p, grid, st);
+    case 256: return km ? launch_one<256, tc_max_stages(256, 8, 1), true, kEpiS32, 8, 1>(a, b, o, w, p, grid, st)
+                        : launch_one<256, tc_max_stages(256, 8, 1), false, kEpiS32, 8, 1>(a, b, o, w, p, grid, st);
     case 224:
       if (!km) return cudaErrorInvalidValue;
-      return t ? launch_one<224, tc_max_stages(224, 8, 1), true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-               : launch_one<224, tc_max_stages(224, 8, 0), true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
+      return t ? launch_one<224, tc_max_stages(224, 8, 1), true, kEpiS32, 8, 1>(a, b, o, w, p, grid, st)
+               : launch_one<224, tc_max_stages(224, 8, 0), true, kEpiS32, 8, 0>(a, b, o, w, p, grid, st);
     case 192:
       if (km)
-        return t ? launch_one<192, tc_max_stages(192, 8, 1), true, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-                 : launch_one<192, tc_max_stages(192, 8, 0), true, kEpiS32, 8, 0>(a, b, o, p, grid, st);
-      return t ? launch_one<192, tc_max_stages(192, 8, 1), false, kEpiS32, 8, 1>(a, b, o, p, grid, st)
-               : launch_one<192, tc_max_stages(192, 8, 0), false, kEpiS32, 8, 0>(a, b, o, p, grid, st);
-    case 128: return km ? launch_one<128, tc_max_stages(128, 4, 1), true, kEpiS32, 4, 1>(a, b, o, p, grid, st)
-                        : launch_one<128, tc_max_stages(128, 4, 1), false, kEpiS32, 4, 1>(a, b, o, p, grid, st);
+        return t ? launch_one<192, tc_max_stages(192, 8, 1), true, kEpiS32, 8, 1>(a, b, o, w, p, grid, st)
+                 : launch_one<192, tc_max_stages(192, 8, 0), true, kEpiS32, 8, 0>(a, b, o, w, p, grid, st);
+      return t ? launch_one<192, tc_max_stages(192, 8, 1), false, kEpiS32, 8, 1>(a, b, o, w, p, grid, st)
+               : launch_one<192, tc_max_stages(192, 8, 0), false, kEpiS32, 8, 0>(a, b, o, w, p, grid, st);
+    case 128: return km ? launch_one<128, tc_max_stages(128, 4, 1), true, kEpiS32, 4, 1>(a, b, o, w, p, grid, st)
+                        : launch_one<128, tc_max_stages(128, 4, 1), false, kEpiS32, 4, 1>(a, b, o, w, p, grid, st);
   }
   return cudaErrorInvalidValue;
 }

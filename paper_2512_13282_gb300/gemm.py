@@ -40,7 +40,7 @@ GEMM_ROUTE_TINY = 6
 class gemm_plan_t(ctypes.Structure):
     _fields_ = [("route", ctypes.c_int), ("bn", ctypes.c_int), ("splits", ctypes.c_int),
                 ("stages", ctypes.c_int), ("grid", ctypes.c_int), ("model_us", ctypes.c_double),
-                ("dram_us", ctypes.c_double)]
+                ("dram_us", ctypes.c_double), ("tail_splits", ctypes.c_int)]
 
 _lock = threading.Lock()
 _lib = None
@@ -171,7 +171,7 @@ def gemm_selftest_wait_timeout(limit_ns: int, stream=None) -> int:
 
 def gemm_plan_query(M, N, K, int8, b_layout, sms=152, pair_slots=76):
     """(status, plan) of the host-only planner query; plan is a dict with
-    route, bn, splits, stages, grid, model_us and dram_us."""
+    route, bn, splits, stages, grid, model_us, dram_us and tail_splits."""
     out = gemm_plan_t()
     st = int(library().gemm_plan_query(M, N, K, 1 if int8 else 0, int(b_layout), int(sms), int(pair_slots),
                                        ctypes.byref(out)))

@@ -199,10 +199,13 @@ def plan_widths(dtype, pair, b_kmajor):
 
 
 def candidate_plans(M, N, K, dtype, b_kmajor, sms=None, pair_slots=None):
-    """Every (family, BN, S) the planner considers for an M x N x K GEMM,
-    with its tile count, K steps per unit and rounds.  Pairs need M > 128;
-    tiles wider than 128 only where N > 128; S keeps >= 4 K steps per unit
-    and at most 2 units per slot."""
+    """Every (family, BN, S, tail split) the planner considers for an
+    M x N x K GEMM, with its tile count, K steps per unit and rounds.  Pairs
+    need M > 128; tiles wider than 128 only where N > 128; S keeps >= 4 K
+    steps per unit and at most 2 units per slot.  After the splits of each
+    width come its split-tail plans: whole tiles for the full rounds, the
+    tiles of a last, partly filled round split in T = 2 .. 8 (tail x T at
+    most one round, >= 4 K steps a unit)."""
     sms = sms or GB300["sms"]
     pair_slots = pair_slots if pair_slots is not None else GB300["pair_slots"]
     num_kb = _ceil(K, BK)
@@ -226,8 +229,35 @@ def candidate_plans(M, N, K, dtype, b_kmajor, sms=None, pair_slots=None):
                     continue
                 seen.add(s2)
                 out.append({"pair": pair, "bn": bn, "splits": s2, "kb_per": kb_per, "tiles": tiles,
-                            "rounds": _ceil(tiles * s2, slots)})
+                            "rounds": _ceil(tiles * s2, slots), "tail_splits": 0})
+            full, tail = divmod(tiles, slots)
+            if full < 1 or tail == 0:
+                continue
+            for t in range(2, 9):
+                if tail * t > slots:
+                    break
+                kb_tail = _ceil(num_kb, t)
+                if _ceil(num_kb, kb_tail) != t or kb_tail < 4:
+                    continue
+                out.append({"pair": pair, "bn": bn, "splits": 1, "kb_per": num_kb, "tiles": tiles,
+                            "rounds": full + 1, "tail_splits": t, "kb_tail": kb_tail, "tail": tail})
     return out
+
+
+def plan_terms(M, N, plan):
+    """(K steps, units) of the busiest CTA and MB of split-K partials of a
+    plan: rounds x kb_per steps with split-K; the full rounds' steps plus one
+    tail unit's with a split tail, whose partials cover only the tail tiles."""
+    if plan.get("tail_splits", 0):
+        rows = 2 * BM if plan["pair"] else BM
+        steps = (plan["rounds"] - 1) * plan["kb_per"] + plan["kb_tail"]
+        return steps, plan["rounds"], 4 * plan["tail_splits"] * plan["tail"] * rows * plan["bn"] / 1e6
+    mb = 4 * plan["splits"] * M * N / 1e6 if plan["splits"] > 1 else 0.0
+    return plan["rounds"] * plan["kb_per"], plan["rounds"], mb
+
+
+def plan_key(plan):
+    return (plan["pair"], plan["bn"], plan["splits"], plan.get("tail_splits", 0))
 
 
 # ------------------------------------------------------------------ cost
@@ -258,11 +288,12 @@ def plan_cost_us(M, N, K, dtype, plan, table):
     g = table["groups"].get(group_key(dtype, plan["pair"], plan["bn"]))
     if g is None:
         return math.inf
-    t_comp = plan["rounds"] * (plan["kb_per"] * g["kstep_us"] + g["unit_us"])
+    steps, rounds, mb = plan_terms(M, N, plan)
+    t_comp = steps * g["kstep_us"] + rounds * g["unit_us"]
     t_split = 0.0
-    if plan["splits"] > 1:
+    if mb > 0:
         sp = table["split"][dtype]
-        t_split = sp["fixed_us"] + sp["us_per_mb"] * 4 * plan["splits"] * M * N / 1e6
+        t_split = sp["fixed_us"] + sp["us_per_mb"] * mb
     return t_comp + t_split
 
 
@@ -322,11 +353,12 @@ def fit(meas):
             r[d] = 1.0
             r[2] = staging_mb(s["M"], s["N"], s["K"], s["dtype"])
             gi = gidx[group_key(s["dtype"], p["pair"], p["bn"])]
-            r[base + 2 * gi] = p["rounds"] * p["kb_per"]
-            r[base + 2 * gi + 1] = p["rounds"]
-            if p["splits"] > 1:
+            steps, rounds, mb = plan_terms(s["M"], s["N"], p)
+            r[base + 2 * gi] = steps
+            r[base + 2 * gi + 1] = rounds
+            if mb > 0:
                 r[base + 2 * ng + 2 * d] = 1.0
-                r[base + 2 * ng + 2 * d + 1] = 4 * p["splits"] * s["M"] * s["N"] / 1e6
+                r[base + 2 * ng + 2 * d + 1] = mb
             rows.append(r)
             rhs.append(p["us"])
             weights.append(1.0 / math.sqrt(best))
@@ -387,13 +419,12 @@ def evaluate(meas, table):
     rep = []
     for s in meas["shapes"]:
         choice = choose_plan(s["M"], s["N"], s["K"], s["dtype"], s["layout"] == "col", table, meas.get("sms"))
-        by = {(p["pair"], p["bn"], p["splits"]): p["us"] for p in s["plans"]}
+        by = {plan_key(p): p["us"] for p in s["plans"]}
         best = min(s["plans"], key=lambda p: p["us"])
         rep.append({"shape": f"{s['dtype']} {s['M']}x{s['N']}x{s['K']} {s['layout']}",
-                    "model_us": by.get((choice["pair"], choice["bn"], choice["splits"])),
+                    "model_us": by.get(plan_key(choice)),
                     "planner_us": s["planner_us"], "best_us": best["us"],
-                    "model_choice": (choice["pair"], choice["bn"], choice["splits"]),
-                    "best": (best["pair"], best["bn"], best["splits"])})
+                    "model_choice": plan_key(choice), "best": plan_key(best)})
     return rep
 
 

@@ -5,7 +5,7 @@ starting values and each step's efficiency are measured on the device).  For
 each shape of a fixed set -- the tensor-core GEMMs of the benchmark
 workloads and a seeded sample of the roofline sweep sizes -- every plan the
 library can be forced into (kernel family: one CTA per 128-row tile or a CTA
-pair per 256-row tile; tile width BN; split-K factor S) is timed with CUDA
+pair per 256-row tile; tile width BN; split-K factor S; split tail T) is timed with CUDA
 events after a 512 MiB L2 flush: the mean of `reps` launches without the
 fastest and the slowest (the event clock advances in steps of about 1 us on
 GB300, so a median of a few launches of a 10-30 us GEMM is off by up to a
@@ -32,8 +32,8 @@ import numpy as np
 from . import workloads as W
 from .tile_model import candidate_plans, GB300
 
-ENV_KEYS = ("GB300_GEMM_BN", "GB300_GEMM_PAIR", "GB300_GEMM_SPLITS", "GB300_GEMM_SKINNY_MAX_M",
-            "GB300_GEMM_S8TM", "GB300_GEMM_TINY_MAX_MACS")
+ENV_KEYS = ("GB300_GEMM_BN", "GB300_GEMM_PAIR", "GB300_GEMM_SPLITS", "GB300_GEMM_TAIL_SPLITS",
+            "GB300_GEMM_SKINNY_MAX_M", "GB300_GEMM_S8TM", "GB300_GEMM_TINY_MAX_MACS")
 # every int8 GEMM of the sweep on the tensor-core kernels
 TC_ONLY = {"GB300_GEMM_SKINNY_MAX_M": 0, "GB300_GEMM_S8TM": 0, "GB300_GEMM_TINY_MAX_MACS": 0}
 
@@ -126,11 +126,12 @@ def main(argv=None):
         plans = []
         for c in candidate_plans(M, N, K, dtype, layout == W.B_COL_MAJOR, sms=sms, pair_slots=GB300["pair_slots"]):
             setenv(dict(TC_ONLY, GB300_GEMM_PAIR=int(c["pair"]), GB300_GEMM_BN=c["bn"],
-                        GB300_GEMM_SPLITS=c["splits"]))
+                        GB300_GEMM_SPLITS=c["splits"], GB300_GEMM_TAIL_SPLITS=c["tail_splits"]))
             plans.append(dict(c, us=round(time_plan(M, N, K, dtype, layout), 3)))
         best = min(plans, key=lambda p: p["us"])
         print(f"{dtype:4s} {M}x{N}x{K} {'col' if layout else 'row'}: planner {default_us:8.1f} us, best forced "
-              f"{best['us']:8.1f} ({'pair' if best['pair'] else 'single'} BN={best['bn']} S={best['splits']})",
+              f"{best['us']:8.1f} ({'pair' if best['pair'] else 'single'} BN={best['bn']} S={best['splits']} "
+              f"T={best['tail_splits']})",
               file=sys.stderr, flush=True)
         rows.append({"M": M, "N": N, "K": K, "dtype": dtype, "layout": "col" if layout else "row",
                      "planner_us": round(default_us, 3), "plans": plans})

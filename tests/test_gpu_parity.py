@@ -355,6 +355,41 @@ def test_parity_narrow_bf16_tiles(layout, bn, monkeypatch):
         _check("bf16", A, B, layout, C)
 
 
+SPLIT_TAIL = [  # (M, N, K, BN, pair, T): 165 = 152 + 13 tiles, 81 = 76 + 5 pairs
+    (1300, 1900, 777, 128, "0", 2), (1300, 1901, 2500, 128, "0", 3),
+    (2100, 2300, 1000, 256, "1", 2), (2100, 2303, 2500, 256, "1", 4),
+]
+
+
+@pytest.mark.parametrize("dtype", ["int8", "bf16", "int8_int16"])
+@pytest.mark.parametrize("layout", [ROW, COL], ids=["Brow", "Bcol"])
+@pytest.mark.parametrize("M,N,K,bn,pair,T", SPLIT_TAIL,
+                         ids=[f"{m}x{n}x{k}-bn{b}-{'pair' if p == '1' else 'single'}-T{t}"
+                              for m, n, k, b, p, t in SPLIT_TAIL])
+def test_parity_split_tail(dtype, layout, M, N, K, bn, pair, T, monkeypatch):
+    """Split tail: the tiles of the last, partly filled round are split in T
+    K ranges (crossing int8 1024-deep slabs) that write partials, reduced
+    over those tiles only, while every other tile writes C -- ragged edges,
+    N with rows not ending on a 16-byte boundary (partials stored directly),
+    TMA and direct stores (GB300_GEMM_TMA_STORE=0), int16 requantisation;
+    the plan query reports the split tail."""
+    monkeypatch.setenv("GB300_GEMM_BN", str(bn))
+    monkeypatch.setenv("GB300_GEMM_PAIR", pair)
+    monkeypatch.setenv("GB300_GEMM_TAIL_SPLITS", str(T))
+    G.gemm_reload_overrides()
+    st, plan = G.gemm_plan_query(M, N, K, dtype != "bf16", layout)
+    assert st == 0 and plan["tail_splits"] == T and plan["splits"] == 1 and plan["bn"] == bn, plan
+    src = "bf16" if dtype == "bf16" else "int8"
+    A, B = _inputs(src, M, N, K, layout, seed=M + N + K + T)
+    for tma in ("1", "0"):
+        monkeypatch.setenv("GB300_GEMM_TMA_STORE", tma)
+        if dtype == "int8_int16":
+            C = U.run(dtype, A, B, layout, shift=5)
+            assert np.array_equal(C.astype(np.int64), oracle.requantize(oracle.gemm_s8(A, B, layout), 5, 16))
+        else:
+            _check(src, A, B, layout, U.run(dtype, A, B, layout))
+
+
 SKINNY = [(1, 1, 1), (1, 11008, 4096), (2, 257, 777), (3, 1000, 4100), (5, 300, 64), (8, 4096, 4096),
           (13, 555, 2049), (16, 4096, 4096), (16, 96, 20000)]
 

@@ -15,7 +15,7 @@ from paper_2512_13282_gb300 import build as B
 from paper_2512_13282_gb300 import gemm as G
 from paper_2512_13282_gb300 import tile_model as T
 
-OVERRIDES = ("GB300_GEMM_BN", "GB300_GEMM_PAIR", "GB300_GEMM_SPLITS", "GB300_GEMM_SKINNY_MAX_M",
+OVERRIDES = ("GB300_GEMM_BN", "GB300_GEMM_PAIR", "GB300_GEMM_SPLITS", "GB300_GEMM_TAIL_SPLITS", "GB300_GEMM_SKINNY_MAX_M",
              "GB300_GEMM_S8TM", "GB300_GEMM_TMA_STORE", "GB300_GEMM_TINY_MAX_MACS")
 
 
@@ -116,8 +116,8 @@ def test_library_planner_equals_the_model(lib):
         if plan["route"] not in (G.GEMM_ROUTE_TC_SINGLE, G.GEMM_ROUTE_TC_PAIR):
             continue
         want = T.choose_plan(M, N, K, dtype, layout == 1, table)
-        got = (plan["route"] == G.GEMM_ROUTE_TC_PAIR, plan["bn"], plan["splits"])
-        assert got == (want["pair"], want["bn"], want["splits"]), (M, N, K, dtype, layout, plan, want)
+        got = (plan["route"] == G.GEMM_ROUTE_TC_PAIR, plan["bn"], plan["splits"], plan["tail_splits"])
+        assert got == T.plan_key(want), (M, N, K, dtype, layout, plan, want)
         assert plan["model_us"] == pytest.approx(T.plan_cost_us(M, N, K, dtype, want, table), rel=1e-4)
         assert plan["dram_us"] == pytest.approx(T.mem_time_us(M, N, K, dtype, want), rel=1e-6)
         checked += 1
@@ -181,10 +181,10 @@ def test_balanced_search_on_the_measurements():
     table = T.fit(meas)
     close, steps = 0, []
     for s in meas["shapes"]:
-        by = {(p["pair"], p["bn"], p["splits"]): p["us"] for p in s["plans"]}
+        by = {T.plan_key(p): p["us"] for p in s["plans"]}
         best = min(by.values())
         plan, t, n = T.balanced_search(s["M"], s["N"], s["K"], s["dtype"], s["layout"] == "col",
-                                       lambda p: by.get((p["pair"], p["bn"], p["splits"]), float("inf")), table,
+                                       lambda p: by.get(T.plan_key(p), float("inf")), table,
                                        meas.get("sms"))
         steps.append(n)
         close += t <= 1.05 * best
