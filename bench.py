@@ -429,7 +429,9 @@ def run_ours(args, rank, world, dev):
                   "to issue a step on the host", file=sys.stderr)
         # The results that came back through the row blocks equal those of
         # one whole-matrix call (int8: bit for bit; bf16: the blocks may
-        # split K differently, so within a bf16 rounding step).
+        # split K differently, so each is within the accumulation bound of
+        # the exact sum -- 2^-8 of it plus 2^-20 of the sum of |a b| -- and
+        # they are within twice that of each other).
         for c in e2e_cases:
             c.launch()
             whole = c.C.cpu()
@@ -437,7 +439,11 @@ def run_ours(args, rank, world, dev):
             if c.g.dtype == "bf16":
                 a = whole.view(torch.bfloat16).float()
                 b = got.view(torch.bfloat16).float()
-                ok = bool(torch.all((a - b).abs() <= 2.0 ** -7 * torch.maximum(a.abs(), b.abs())))
+                a_abs = c.A.view(torch.bfloat16).float().abs()
+                b_abs = c.B.view(torch.bfloat16).float().abs()
+                mag = (a_abs @ (b_abs if c.g.layout == W.B_ROW_MAJOR else b_abs.t())).cpu()
+                del a_abs, b_abs
+                ok = bool(torch.all((a - b).abs() <= 2.0 ** -7 * torch.maximum(a.abs(), b.abs()) + 2.0 ** -19 * mag))
             else:
                 ok = torch.equal(whole, got)
             if not ok:
