@@ -461,9 +461,10 @@ def header_text(table, source="plan_measurements.json"):
         "// BK = 64 (eff of Eq. 1 measured) and the fixed time of one unit (start and",
         "// epilogue), in microseconds; and per operand type the split-K terms",
         "// (reduction launch, and time per MB of fp32/int32 partials).  The planner",
-        "// minimises rounds * (K steps per unit * kstep + unit) + split terms",
-        "// (Eq. 9 with wave quantisation) + kMemWeight * the DRAM time of Eq. 6-8,",
-        "// 10 (the share of B's re-reads the kernels do not hide).",
+        "// minimises the busiest CTA's K steps * kstep + its units * unit + split",
+        "// terms (Eq. 9 with wave quantisation; a split tail adds one round of a",
+        "// tail unit's steps to the full rounds) + kMemWeight * the DRAM time of",
+        "// Eq. 6-8, 10 (the share of B's re-reads the kernels do not hide).",
         "#pragma once",
         "",
         "namespace gb300 {",
