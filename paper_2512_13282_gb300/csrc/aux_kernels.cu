@@ -183,7 +183,8 @@ __global__ void zero_fill_kernel(T *C, int64_t M, int64_t N, int64_t ldc) {
 // C's address allows it.
 struct Piece {
   int64_t r, c;
-  int n;  // elements in the piece (4, or fewer at the end of a row)
+  int n;      // elements in the piece (4, or fewer at the end of a row)
+  int64_t w;  // offset of its first element in a plane of partials
 };
 
 __device__ __forceinline__ Piece piece_of(uint64_t t, uint32_t cpr, int64_t N) {
@@ -199,10 +200,14 @@ __device__ __forceinline__ Piece piece_of(uint64_t t, uint32_t cpr, int64_t N) {
   pc.r = (int64_t)r;
   pc.c = (int64_t)q * 4;
   pc.n = N - pc.c < 4 ? (int)(N - pc.c) : 4;
+  pc.w = pc.r * N + pc.c;
   return pc;
 }
 
 // Piece t of the part of C that rt covers; false when it lies outside C.
+// Partials of all of C are planes of C's shape; those of a split tail are
+// compact: per plane, tile i of the tail as rows x cols words at row
+// i * rows.
 __device__ __forceinline__ bool reduce_piece(uint64_t t, uint32_t cpr, int64_t M, int64_t N, const ReduceTiles &rt,
                                              Piece *pc) {
   if (rt.count == 0) {
@@ -217,20 +222,24 @@ __device__ __forceinline__ bool reduce_piece(uint64_t t, uint32_t cpr, int64_t M
   const uint32_t rem = (uint32_t)(t - (uint64_t)ti * per_tile);
   int tm, tn;
   raster_tile(rt.first + ti, rt.tiles_m, rt.tiles_n, rt.group_m, &tm, &tn);
-  pc->r = (int64_t)tm * rt.rows + rem / cpt;
-  pc->c = (int64_t)tn * rt.cols + (int64_t)(rem % cpt) * 4;
+  const uint32_t rl = rem / cpt, cl = (rem % cpt) * 4;
+  pc->r = (int64_t)tm * rt.rows + rl;
+  pc->c = (int64_t)tn * rt.cols + cl;
   if (pc->r >= M || pc->c >= N) return false;
   pc->n = N - pc->c < 4 ? (int)(N - pc->c) : 4;
+  pc->w = ((int64_t)ti * rt.rows + rl) * rt.cols + cl;
   return true;
 }
 
+// Sum of a piece over the planes (plane stride MN words); vec: the
+// pieces of a plane start on 16-byte boundaries.
 template <typename T>
-__device__ __forceinline__ void sum_piece(const T *__restrict__ ws, int splits, int64_t MN, int64_t N,
+__device__ __forceinline__ void sum_piece(const T *__restrict__ ws, int splits, int64_t MN, bool vec,
                                           const Piece &pc, T (&v)[4]) {
-  const int64_t base = pc.r * N + pc.c;
+  const int64_t base = pc.w;
 #pragma unroll
   for (int i = 0; i < 4; ++i) v[i] = T(0);
-  if (pc.n == 4 && (N & 3) == 0) {
+  if (pc.n == 4 && vec) {
     for (int k = 0; k < splits; ++k) {
       const uint4 w = __ldcs(reinterpret_cast<const uint4 *>(ws + (int64_t)k * MN + base));
       T x[4];
@@ -252,7 +261,8 @@ __global__ void __launch_bounds__(kThreads)
   Piece pc;
   if (!reduce_piece(t, cpr, M, N, rt, &pc)) return;
   float v[4];
-  sum_piece(ws, splits, M * N, N, pc, v);
+  sum_piece(ws, splits, rt.count ? (int64_t)rt.count * rt.rows * rt.cols : M * N,
+            rt.count ? true : (N & 3) == 0, pc, v);
   uint16_t *dst = C + pc.r * ldc + pc.c;
   uint16_t h[4];
 #pragma unroll
@@ -276,7 +286,8 @@ __global__ void __launch_bounds__(kThreads)
   Piece pc;
   if (!reduce_piece(t, cpr, M, N, rt, &pc)) return;
   int32_t v[4];
-  sum_piece(ws, splits, M * N, N, pc, v);
+  sum_piece(ws, splits, rt.count ? (int64_t)rt.count * rt.rows * rt.cols : M * N,
+            rt.count ? true : (N & 3) == 0, pc, v);
   if (out_bits == 32) {
     int32_t *dst = static_cast<int32_t *>(C) + pc.r * ldc + pc.c;
     if (pc.n == 4 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0)

@@ -548,9 +548,23 @@ struct WsLayout {
   size_t a_off = 0, b_off = 0, part_off = 0, total = 0;
 };
 
-// Planes of M x N 32-bit partials a plan writes (split-K, or a split tail,
-// which writes only its tiles' parts of them); 0 when C is written directly.
+// Planes of 32-bit partials a plan writes (split-K, or a split tail); 0 when
+// C is written directly.
 int64_t partial_planes(const TcParams &p) { return p.splits > 1 ? p.splits : p.tail_splits; }
+
+// Rows of one plane of a split tail's compact partials (the tail tiles'
+// rows one after the other; row pitch BN).
+int64_t tail_rows(const Plan &pl) {
+  return (int64_t)(pl.p.tiles_m * pl.p.tiles_n - pl.p.tail_first) * (pl.v.pair ? 2 * kBM : kBM);
+}
+
+// Bytes of partials: planes of C's shape for split-K, compact blocks of the
+// tail tiles for a split tail.
+size_t partial_bytes(const Plan &pl) {
+  if (pl.p.splits > 1) return (size_t)pl.p.splits * pl.p.M * pl.p.N * 4;
+  if (pl.p.tail_splits > 0) return (size_t)pl.p.tail_splits * tail_rows(pl) * pl.v.bn * 4;
+  return 0;
+}
 
 // Shared path after staging: encode maps, launch the tcgen05 kernel and the
 // split-K reduction.
@@ -588,10 +602,11 @@ gemm_status_t run_tc(DeviceState &d, Plan &pl, const uint16_t *A, int64_t lda, c
   CUtensorMap tout = tb, tws = tb;
   p.out_tma = kOutDirect;
   p.ws_tma = 0;
-  // a split tail's partials go through TMA where split-K partials would
-  if (p.tail_splits > 0 && pl.v.tma_out == 1 && p.N % 4 == 0 && overrides().tma_store) {
+  // a split tail's compact partials go through TMA in the variants with
+  // 4 KB staging blocks (their rows, BN words, always end on 16 bytes)
+  if (p.tail_splits > 0 && pl.v.tma_out == 1 && overrides().tma_store) {
     if (!encode_out(&tws, s32 ? CU_TENSOR_MAP_DATA_TYPE_INT32 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, partials,
-                    (uint64_t)p.N, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.tail_splits))
+                    (uint64_t)pl.v.bn, (uint64_t)tail_rows(pl), (uint64_t)pl.v.bn, (uint64_t)p.tail_splits))
       return cuda_failed("tail partials tensor map");
     p.ws_tma = 1;
   }
@@ -738,7 +753,7 @@ gemm_status_t gemm_bf16_f32acc_bf16(int64_t M, int64_t N, int64_t K, const uint1
   if (pack_b) { L.b_off = off; off = align_up(off + (size_t)b_rows * ldb_p * 2, 256); }
   if (partial_planes(pl.p) > 0) {
     L.part_off = off;
-    off = align_up(off + (size_t)partial_planes(pl.p) * M * N * 4, 256);
+    off = align_up(off + partial_bytes(pl), 256);
   }
   L.total = off;
   if (L.total && (s = ensure_workspace(L.total, st)) != GEMM_OK) return s;
@@ -987,7 +1002,7 @@ gemm_status_t s8_gemm(int64_t M, int64_t N, int64_t K, const int8_t *A, int64_t 
   off = align_up(off + (size_t)b_rows * ldb_p * 2, 256);
   if (partial_planes(pl.p) > 0) {
     L.part_off = off;
-    off = align_up(off + (size_t)partial_planes(pl.p) * M * N * 4, 256);
+    off = align_up(off + partial_bytes(pl), 256);
   }
   L.total = off;
   if ((s = ensure_workspace(L.total, st)) != GEMM_OK) return s;
@@ -1191,8 +1206,7 @@ gemm_status_t s8_gemm_into_scratch(int64_t M, int64_t N, int64_t K, const int8_t
   const size_t b_off = align_up((size_t)M * lda_p * 2, 256);
   const size_t part_off = align_up(b_off + (size_t)b_rows * ldb_p * 2, 256);
   auto total_of = [&](const Plan &q) {
-    const int64_t planes = partial_planes(q.p);
-    return planes > 0 ? align_up(part_off + (size_t)planes * M * N * 4, 256) : part_off;
+    return partial_planes(q.p) > 0 ? align_up(part_off + partial_bytes(q), 256) : part_off;
   };
   // a split tail's partial planes may not fit the caller's scratch: plan
   // without one then

@@ -65,7 +65,7 @@ struct TcParams {
   void *C;           // bf16 or int32 output, row-major, leading dimension ldc
   int64_t ldc;
   int c_vec;         // C rows 16-byte aligned (informational; stores check each address)
-  void *ws;          // split-K partials, splits x M x N 32-bit words (fp32 or int32)
+  void *ws;          // partials (fp32 or int32): split-K, splits x M x N words; a split tail, compact (below)
   uint32_t *err;     // device error word
   uint64_t wait_limit_ns;
   int out_bits;      // int8 path: 32 (exact int32 C), 16 or 8 (requantised C)
@@ -73,11 +73,13 @@ struct TcParams {
   int out_tma;       // kOutDirect, kOutTmaC (tmOut maps C) or kOutTmaWs (tmOut maps the partials)
   // Split tail (tail_splits >= 2, splits == 1): the tiles of the last,
   // partly filled round -- raster positions tail_first .. -- are each split
-  // into tail_splits units of tail_kb_per k-blocks that write partials
-  // (planes as for split-K) for the reduction kernel, so that the round
-  // takes 1 / tail_splits of a tile's time; every other tile is one unit
-  // writing C.  tail_first is a whole number of rounds of units.  ws_tma:
-  // the partials are stored through tmWs (else directly).
+  // into tail_splits units of tail_kb_per k-blocks that write partials for
+  // the reduction kernel, so that the round takes 1 / tail_splits of a
+  // tile's time; every other tile is one unit writing C.  tail_first is a
+  // whole number of rounds of units.  The tail's partials are compact:
+  // plane s holds, for the tail tile at raster position tail_first + i, a
+  // block of tile rows x BN 32-bit words at row i * tile rows (row pitch BN).
+  // ws_tma: they are stored through tmWs (else directly).
   int tail_first, tail_splits, tail_kb_per, ws_tma;
 };
 
@@ -139,6 +141,7 @@ struct TcCfg {
 struct Unit {
   int tm, tn, split, kb0, kb1;
   int part;  // 1: the unit writes split-K partials (plane `split`), 0: C
+  int slot;  // split-tail units: the tile's place among the tail tiles
 };
 
 // Raster position t -> output tile (tm, tn).  Tiles are visited in groups of
@@ -178,7 +181,9 @@ __device__ __forceinline__ Unit decode_unit(const TcParams &p, int u) {
     w.kb0 = w.split * p.tail_kb_per;
     w.kb1 = min(p.num_kb, w.kb0 + p.tail_kb_per);
     w.part = 1;
+    w.slot = t - p.tail_first;
   } else {
+    w.slot = 0;
     w.split = u / num_tiles;
     t = u - w.split * num_tiles;
     w.kb0 = w.split * p.kb_per_split;
@@ -435,17 +440,18 @@ __device__ __forceinline__ void tma_out_narrow(const CUtensorMap *tm, uint32_t b
 // else directly.
 __device__ __forceinline__ void store_s32_chunk(const TcParams &p, const CUtensorMap *tm, uint32_t ebuf, int lane,
                                                 int out_tma, const uint32_t (&v)[32], int x, int y0, int split,
-                                                bool row_ok, int64_t row, uint32_t *wrow, bool ws_vec) {
+                                                bool row_ok, int64_t row, uint32_t *wrow, bool ws_vec, int px,
+                                                int py, int pn) {
   if (out_tma != kOutDirect) {
     if (out_tma == kOutTmaWs)
-      tma_out_words32<true>(tm, ebuf, lane, v, x, y0, split, y0 < p.M && x < p.N);
+      tma_out_words32<true>(tm, ebuf, lane, v, x - px, y0 - py, split, y0 < p.M && x < p.N);
     else if (p.out_bits == 32)
       tma_out_words32<false>(tm, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
     else
       tma_out_narrow(tm, ebuf, lane, v, p.out_bits, p.out_shift, x, y0, y0 < p.M && x < p.N);
   } else if (row_ok) {
     if (wrow)
-      store_words<32>(wrow, x, p.N, ws_vec, v);
+      store_words<32>(wrow, x - px, pn, ws_vec, v);
     else
       store_s8_result<32>(p, row, x, v);
   }
@@ -615,6 +621,13 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
       const bool tail = split && p.tail_splits > 0;    // ... of a split-tail tile
       const int uo = tail ? tail_out : out_tma;
       const CUtensorMap *om = tail ? &tmWs : &tmOut;
+      // partial coordinates: a split-tail tile's partials are a compact
+      // block (origin px, py of the matrix; rows of pn words), split-K
+      // partials whole planes of C's shape
+      const int px = tail ? w.tn * BN : 0;
+      const int py = tail ? (w.tm - w.slot) * kBM : 0;
+      const int pn = tail ? BN : p.N;
+      const int64_t pm = tail ? (int64_t)(p.tiles_m * p.tiles_n - p.tail_first) * kBM : (int64_t)p.M;
       const int64_t row = (int64_t)w.tm * kBM + row_in_tile;
       const bool row_ok = row < p.M;
       const int col0 = w.tn * BN + colpart * CPT;
@@ -631,7 +644,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
           }
           tc_fence_after_sync();
           const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
-          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+          uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * pm + (row - py)) * pn
                                  : nullptr;
 #pragma unroll 1
           for (int c = 0; c < CPT / 32; ++c) {
@@ -640,7 +653,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
             tmem_ld_wait();
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(__float2int_rn(__uint_as_float(v[i])));
-            store_s32_chunk(p, om, ebuf, lane, uo, v, col0 + c * 32, y0, w.split, row_ok, row, wrow, ws_vec);
+            store_s32_chunk(p, om, ebuf, lane, uo, v, col0 + c * 32, y0, w.split, row_ok, row, wrow, ws_vec, px, py, pn);
           }
           if constexpr (CPT % 32 != 0) {  // a 16-column tail: each lane stores its row
             constexpr int kTail = (CPT / 32) * 32;
@@ -651,7 +664,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
             for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(__float2int_rn(__uint_as_float(v[i])));
             if (row_ok) {
               if (split)
-                store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+                store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, v);
               else
                 store_s8_result<16>(p, row, col0 + kTail, v);
             }
@@ -695,7 +708,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
         }
         if (!ok) break;
         // split-K partials stay int32; the reduction requantises
-        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * pm + (row - py)) * pn
                                : nullptr;
         if (uo != kOutDirect) {
 #pragma unroll
@@ -705,7 +718,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
             const int x = col0 + c * 32;
             if (uo == kOutTmaWs)
-              tma_out_words32<true>(om, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
+              tma_out_words32<true>(om, ebuf, lane, v, x - px, y0 - py, w.split, y0 < p.M && x < p.N);
             else if (p.out_bits == 32)
               tma_out_words32<false>(om, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
             else
@@ -718,7 +731,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
 #pragma unroll
               for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
               if (split)
-                store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+                store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, v);
               else
                 store_s8_result<16>(p, row, col0 + kTail, v);
             }
@@ -730,7 +743,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
             if (split)
-              store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, v);
+              store_words<32>(wrow, col0 + c * 32 - px, pn, ws_vec, v);
             else
               store_s8_result<32>(p, row, col0 + c * 32, v);
           }
@@ -740,7 +753,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
             if (split)
-              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+              store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, v);
             else
               store_s8_result<16>(p, row, col0 + kTail, v);
           }
@@ -754,7 +767,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
         tc_fence_after_sync();
         const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
         uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
-        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * pm + (row - py)) * pn
                                : nullptr;
 #pragma unroll 1
         for (int c = 0; c < CPT / 32; ++c) {
@@ -763,14 +776,14 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
           tmem_ld_wait();
           const int x = col0 + c * 32;
           if (TMA_OUT == 1 && uo == kOutTmaWs) {
-            tma_out_words32<true>(om, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
+            tma_out_words32<true>(om, ebuf, lane, r, x - px, y0 - py, w.split, y0 < p.M && x < p.N);
           } else if (TMA_OUT == 1 && uo == kOutTmaC) {
             tma_out_bf16x32(om, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
           } else if (TMA_OUT == 2 && uo == kOutTmaC) {
             tma_out_bf16x16x2(om, ebuf, lane, r, x, y0, p.M, p.N);
           } else if (row_ok) {
             if (split)
-              store_words<32>(wrow, x, p.N, ws_vec, r);
+              store_words<32>(wrow, x - px, pn, ws_vec, r);
             else
               store_bf16<32>(crow, x, p.N, p.c_vec != 0, r);
           }
@@ -782,7 +795,7 @@ __global__ void __launch_bounds__(TcCfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, TM
           tmem_ld_wait();
           if (row_ok) {
             if (split)
-              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, r);
+              store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, r);
             else
               store_bf16<16>(crow, col0 + kTail, p.N, p.c_vec != 0, r);
           }

@@ -282,6 +282,13 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
       const bool tail = split && p.tail_splits > 0;    // ... of a split-tail tile
       const int uo = tail ? tail_out : out_tma;
       const CUtensorMap *om = tail ? &tmWs : &tmOut;
+      // partial coordinates: a split-tail tile's partials are a compact
+      // block (origin px, py of the matrix; rows of pn words), split-K
+      // partials whole planes of C's shape
+      const int px = tail ? w.tn * BN : 0;
+      const int py = tail ? (w.tm - w.slot) * kTileM : 0;
+      const int pn = tail ? BN : p.N;
+      const int64_t pm = tail ? (int64_t)(p.tiles_m * p.tiles_n - p.tail_first) * kTileM : (int64_t)p.M;
       const int64_t row = (int64_t)w.tm * kTileM + row_in_tile;
       const bool row_ok = row < p.M;
       const int col0 = w.tn * BN + colpart * CPT;
@@ -320,7 +327,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
         }
         if (!ok) break;
         // split-K partials stay int32; the reduction requantises
-        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * pm + (row - py)) * pn
                                : nullptr;
         if (uo != kOutDirect) {
 #pragma unroll
@@ -330,7 +337,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
             const int x = col0 + c * 32;
             if (uo == kOutTmaWs)
-              tma_out_words32<true>(om, ebuf, lane, v, x, y0, w.split, y0 < p.M && x < p.N);
+              tma_out_words32<true>(om, ebuf, lane, v, x - px, y0 - py, w.split, y0 < p.M && x < p.N);
             else if (p.out_bits == 32)
               tma_out_words32<false>(om, ebuf, lane, v, x, y0, 0, y0 < p.M && x < p.N);
             else
@@ -343,7 +350,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
 #pragma unroll
               for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
               if (split)
-                store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+                store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, v);
               else
                 store_s8_result<16>(p, row, col0 + kTail, v);
             }
@@ -355,7 +362,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = static_cast<uint32_t>(acc[c * 32 + i]);
             if (split)
-              store_words<32>(wrow, col0 + c * 32, p.N, ws_vec, v);
+              store_words<32>(wrow, col0 + c * 32 - px, pn, ws_vec, v);
             else
               store_s8_result<32>(p, row, col0 + c * 32, v);
           }
@@ -365,7 +372,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] = static_cast<uint32_t>(acc[kTail + i]);
             if (split)
-              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, v);
+              store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, v);
             else
               store_s8_result<16>(p, row, col0 + kTail, v);
           }
@@ -379,7 +386,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
         tc_fence_after_sync();
         const uint32_t t0 = tmem_base + b * BN + ((uint32_t)(quad * 32) << 16) + colpart * CPT;
         uint16_t *crow = reinterpret_cast<uint16_t *>(p.C) + row * p.ldc;
-        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * p.M + row) * p.N
+        uint32_t *wrow = split ? reinterpret_cast<uint32_t *>(p.ws) + ((int64_t)w.split * pm + (row - py)) * pn
                                : nullptr;
 #pragma unroll 1
         for (int c = 0; c < CPT / 32; ++c) {
@@ -388,14 +395,14 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
           tmem_ld_wait();
           const int x = col0 + c * 32;
           if (TMA_OUT == 1 && uo == kOutTmaWs) {
-            tma_out_words32<true>(om, ebuf, lane, r, x, y0, w.split, y0 < p.M && x < p.N);
+            tma_out_words32<true>(om, ebuf, lane, r, x - px, y0 - py, w.split, y0 < p.M && x < p.N);
           } else if (TMA_OUT == 1 && uo == kOutTmaC) {
             tma_out_bf16x32(om, ebuf, lane, r, x, y0, y0 < p.M && x < p.N);
           } else if (TMA_OUT == 2 && uo == kOutTmaC) {
             tma_out_bf16x16x2(om, ebuf, lane, r, x, y0, p.M, p.N);
           } else if (row_ok) {
             if (split)
-              store_words<32>(wrow, x, p.N, ws_vec, r);
+              store_words<32>(wrow, x - px, pn, ws_vec, r);
             else
               store_bf16<32>(crow, x, p.N, p.c_vec != 0, r);
           }
@@ -407,7 +414,7 @@ __global__ void __launch_bounds__(Tc2Cfg<BN, STAGES, B_KMAJOR, EPI, EPI_WARPS, T
           tmem_ld_wait();
           if (row_ok) {
             if (split)
-              store_words<16>(wrow, col0 + kTail, p.N, ws_vec, r);
+              store_words<16>(wrow, col0 + kTail - px, pn, ws_vec, r);
             else
               store_bf16<16>(crow, col0 + kTail, p.N, p.c_vec != 0, r);
           }
