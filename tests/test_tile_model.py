@@ -142,6 +142,27 @@ def test_plan_query_routes(lib):
     assert G.gemm_plan_query(4, 4, 4, True, 2)[0] == G.GEMM_ERR_INVALID_ARG
 
 
+def test_plan_query_split_tail(lib, monkeypatch):
+    """Split tails on the host-only plan query: chosen by the model for
+    8192^3 (1024 CTA-pair tiles on 76 pairs: 13 full rounds and 36 tiles in
+    halves), turned off by GB300_GEMM_TAIL_SPLITS=0, forced to another
+    split count where one fits (T = 3 does not fit 36 pair tiles into 76
+    pairs: a single-CTA width takes it), and absent where the tiles fill no
+    second round."""
+    st, p = G.gemm_plan_query(8192, 8192, 8192, False, 0)
+    assert st == 0 and p["route"] == G.GEMM_ROUTE_TC_PAIR and (p["bn"], p["splits"], p["tail_splits"]) == (256, 1, 2)
+    monkeypatch.setenv("GB300_GEMM_TAIL_SPLITS", "0")
+    G.gemm_reload_overrides()
+    st, p = G.gemm_plan_query(8192, 8192, 8192, False, 0)
+    assert st == 0 and p["tail_splits"] == 0
+    monkeypatch.setenv("GB300_GEMM_TAIL_SPLITS", "3")
+    G.gemm_reload_overrides()
+    st, p = G.gemm_plan_query(8192, 8192, 8192, True, 0)
+    assert st == 0 and p["tail_splits"] == 3 and p["route"] == G.GEMM_ROUTE_TC_SINGLE and p["splits"] == 1
+    st, p = G.gemm_plan_query(1024, 1024, 1024, True, 1)   # 64 tiles: no second round
+    assert st == 0 and p["tail_splits"] == 0
+
+
 def _measurements():
     with open(T.MEASUREMENTS) as f:
         return json.load(f)
